@@ -1,0 +1,181 @@
+"""CPU oracle for the InfiniPot-V compression pass (arXiv 2506.15745).
+
+TEST INFRASTRUCTURE ONLY: imported by tests/, ``__graft_entry__.smoke()`` and
+the cpu_baseline / reference legs of ``bench.py``; never by the product
+package. The arithmetic lives in ``ipv_oracle.cpp`` (plain single-threaded
+C++, fp64); this module compiles it with g++ and marshals numpy arrays.
+
+Functions mirror the paper's steps:
+  scores()  -- TaR (Sec. 3.1, Eq. tar) and VaN (Sec. 3.2) per past token
+  select()  -- split-budget selection (Algorithm 1 steps 3-5, Sec. 3.3)
+  gather()  -- compaction K~ = K[:, J, :] (Sec. 3.1, Algorithm 2 last step)
+  compress()-- the three in sequence (used to time the oracle)
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "ipv_oracle.cpp")
+_LIB = os.path.join(_HERE, "liboracle.so")
+# A prebuilt library to load instead (the mutation tests point this at a copy
+# of the oracle with a planted mistake); never set on the normal path.
+_LIB_OVERRIDE = os.environ.get("IPV_ORACLE_LIB_OVERRIDE")
+_lib = None
+
+
+def build_cmd(src: str = _SRC, out: str = _LIB) -> list[str]:
+    return ["g++", "-O2", "-std=c++17", "-fPIC", "-shared", "-o", out, src]
+
+
+def build(force: bool = False) -> str:
+    """Compile liboracle.so next to its source (no-op when up to date)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        subprocess.run(build_cmd(), check=True)
+    return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        if _LIB_OVERRIDE:
+            lib = ctypes.CDLL(_LIB_OVERRIDE)
+        else:
+            build()
+            lib = ctypes.CDLL(_LIB)
+        P, I64, I32, D = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_double
+        lib.oracle_recent_frames.argtypes = [I64, I32]
+        lib.oracle_recent_frames.restype = I32
+        lib.oracle_scores.argtypes = [P, P, I32, I64, I64, I32, I64, I32, I32, P, P, P]
+        lib.oracle_scores.restype = I32
+        lib.oracle_budget_split.argtypes = [I64, I32, I32, I64, D, P]
+        lib.oracle_budget_split.restype = I32
+        lib.oracle_select.argtypes = [P, P, I64, I64, I32, I32, I64, D, P, P]
+        lib.oracle_select.restype = I32
+        lib.oracle_gather_rows.argtypes = [P, P, I64, I64, I64, I64, P, I64]
+        lib.oracle_gather_rows.restype = I32
+        lib.oracle_gather_patch.argtypes = [P, P, I64, I64, I64, I32, P, I64]
+        lib.oracle_gather_patch.restype = I32
+        lib.oracle_compress.argtypes = [P, P, I32, I64, I64, I32, I64, I32, I32, I64, D,
+                                        P, P, P, P, P]
+        lib.oracle_compress.restype = I32
+        _lib = lib
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _kv_kind(a: np.ndarray) -> int:
+    """1 for bf16 bit patterns (stored as uint16), 0 for float32."""
+    if a.dtype == np.uint16:
+        return 1
+    if a.dtype == np.float32:
+        return 0
+    raise TypeError(f"K/V must be float32 or bf16 bits (uint16), got {a.dtype}")
+
+
+def recent_frames(n_frames: int, override: int = 0) -> int:
+    """r: the override if positive, else max(1, floor(f/8 + 1/2)) (Appendix B.2: r = 0.125 f)."""
+    return _load().oracle_recent_frames(int(n_frames), int(override))
+
+
+def budget_split(n_tokens: int, p: int, r: int, budget: int, alpha: float):
+    """(recent kept, TaR picks, VaN picks); None for the pass-through case."""
+    out = np.zeros(3, np.int64)
+    rc = _load().oracle_budget_split(n_tokens, p, r, budget, float(alpha), _ptr(out))
+    if rc != 0:
+        raise ValueError("no valid budget split for these arguments")
+    return None if out[0] < 0 else tuple(int(x) for x in out)
+
+
+def scores(k: np.ndarray, v: np.ndarray, n_tokens: int, p: int, r: int,
+           patch_id: np.ndarray | None = None):
+    """TaR, VaN in fp64 for K, V of shape [S, cap, D] (float32 or bf16 bits)."""
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    assert k.shape == v.shape and k.dtype == v.dtype and k.ndim == 3
+    S, cap, D = k.shape
+    if patch_id is not None:
+        patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
+        assert patch_id.shape == (S, cap)
+    tar = np.empty((S, n_tokens), np.float64)
+    van = np.empty((S, n_tokens), np.float64)
+    rc = _load().oracle_scores(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
+                               _ptr(patch_id), _ptr(tar), _ptr(van))
+    if rc != 0:
+        raise ValueError("oracle_scores rejected its arguments")
+    return tar, van
+
+
+def select(tar: np.ndarray, van: np.ndarray, n_tokens: int, p: int, r: int, budget: int,
+           alpha: float, with_gaps: bool = False):
+    """kept indices [S, budget] ascending (and per-stage boundary gaps [S, 2])."""
+    tar = np.ascontiguousarray(tar, dtype=np.float64)
+    van = np.ascontiguousarray(van, dtype=np.float64)
+    S = tar.shape[0]
+    assert tar.shape == (S, n_tokens) and van.shape == tar.shape
+    kept = np.empty((S, budget), np.int32)
+    gaps = np.empty((S, 2), np.float64)
+    rc = _load().oracle_select(_ptr(tar), _ptr(van), S, n_tokens, p, r, budget, float(alpha),
+                               _ptr(kept), _ptr(gaps))
+    if rc != 0:
+        raise ValueError("oracle_select rejected its arguments")
+    return (kept, gaps) if with_gaps else kept
+
+
+def gather(src: np.ndarray, kept: np.ndarray, cap_dst: int | None = None,
+           dst: np.ndarray | None = None) -> np.ndarray:
+    """dst[s, j] = src[s, kept[s, j]] (rows with kept == -1 untouched)."""
+    src = np.ascontiguousarray(src)
+    kept = np.ascontiguousarray(kept, dtype=np.int32)
+    S, cap, D = src.shape
+    budget = kept.shape[1]
+    cap_dst = cap if cap_dst is None else cap_dst
+    if dst is None:
+        dst = np.zeros((S, cap_dst, D), src.dtype)
+    rc = _load().oracle_gather_rows(_ptr(src), _ptr(dst), D * src.itemsize, S, cap, cap_dst,
+                                    _ptr(kept), budget)
+    if rc != 0:
+        raise ValueError("oracle_gather_rows rejected its arguments")
+    return dst
+
+
+def gather_patch(src_pid: np.ndarray | None, kept: np.ndarray, p: int, cap_src: int,
+                 cap_dst: int, dst: np.ndarray | None = None) -> np.ndarray:
+    kept = np.ascontiguousarray(kept, dtype=np.int32)
+    S, budget = kept.shape
+    if dst is None:
+        dst = np.zeros((S, cap_dst), np.uint16)
+    if src_pid is not None:
+        src_pid = np.ascontiguousarray(src_pid, dtype=np.uint16)
+    rc = _load().oracle_gather_patch(_ptr(src_pid), _ptr(dst), S, cap_src, cap_dst, p,
+                                     _ptr(kept), budget)
+    if rc != 0:
+        raise ValueError("oracle_gather_patch rejected its arguments")
+    return dst
+
+
+def compress(k: np.ndarray, v: np.ndarray, n_tokens: int, p: int, r: int, budget: int,
+             alpha: float, patch_id: np.ndarray | None = None):
+    """Whole pass: returns (kept [S,budget], K~ [S,cap,D], V~ [S,cap,D], patch ids [S,cap])."""
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    S, cap, D = k.shape
+    kd = np.zeros_like(k)
+    vd = np.zeros_like(v)
+    pd = np.zeros((S, cap), np.uint16)
+    kept = np.empty((S, budget), np.int32)
+    if patch_id is not None:
+        patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
+    rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
+                                 budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
+                                 _ptr(pd), _ptr(kept))
+    if rc != 0:
+        raise ValueError("oracle_compress rejected its arguments")
+    return kept, kd, vd, pd

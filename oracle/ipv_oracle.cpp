@@ -1,0 +1,287 @@
+// InfiniPot-V compression pass: plain CPU oracle (fp64, single-threaded).
+//
+// TEST INFRASTRUCTURE ONLY. Nothing on the product path may link, load or call
+// this file. Its only users are tests/, __graft_entry__.smoke() and the
+// cpu_baseline / reference legs of bench.py. It shares no code, header or
+// constant with the CUDA path (paper_2506_15745_gb300/csrc); the two meet only
+// on the bytes of the synthetic inputs.
+//
+// What it computes, per (layer, KV head) slab, following InfiniPot-V
+// (arXiv 2506.15745):
+//   * TaR score, Sec. 3.1 Eq. (tar): for a past token at frame t, patch (i,j),
+//       s = -(1/r) * sum_{t'=1..r} cos(K_past[t,i,j], K_recent[t',i,j]),
+//     with the cache viewed as f frames of p = |M|/f patches, the r latest
+//     frames "recent" and the rest "past" (Sec. 3.1; Algorithm 2 reshape).
+//     The sum of r cosines is evaluated literally, term by term.
+//   * VaN score, Sec. 3.2: s = ||V[t,i,j]||_2.
+//   * Selection, Algorithm 1 steps (3)-(5) with the Sec. 3.3 split: the r
+//     recent frames are always kept and count inside the TaR share
+//     (alpha*|C| - len(K_recent)); the TaR share is the top of s_TaR over the
+//     past tokens; the rest of |C| is filled by the top of s_VaN over the past
+//     tokens TaR did not take (Algorithm 2 forces TaR picks to max(VaN) before
+//     its final TopK, which is the same as excluding them). Ties go to the
+//     lower token index; NaN scores rank below every number.
+//   * Compaction, Sec. 3.1 / Algorithm 2 last step: K~ = K[:, J, :], the kept
+//     rows copied in ascending index order.
+//
+// Readings where the paper is silent (each is listed in the design notes):
+// alpha*|C| is floored; r defaults to max(1, floor(f/8 + 1/2)) (Appendix B.2
+// standardises r = 0.125 f); a cache at or below |C| tokens is passed through
+// (Algorithm 1 triggers only when len(K) >= |M| > |C|); cosine uses
+// max(||x||, 1e-12) in each denominator so that a zero vector has cosine 0;
+// past-token patch coordinates come from an optional per-token patch-id array
+// (else n mod p), recent rows are whole frames at rows N - r p + t' p + q.
+//
+// Element types: bf16 (widened exactly: bits << 16) or fp32, widened to double.
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <limits>
+#include <vector>
+
+namespace {
+
+double widen(const void* base, int is_bf16, int64_t idx) {
+  if (is_bf16) {
+    uint16_t h = static_cast<const uint16_t*>(base)[idx];
+    uint32_t u = static_cast<uint32_t>(h) << 16;
+    float f;
+    std::memcpy(&f, &u, sizeof f);
+    return static_cast<double>(f);
+  }
+  return static_cast<double>(static_cast<const float*>(base)[idx]);
+}
+
+// Row n of slab s of a [n_slabs][cap][D] tensor, widened to double.
+void load_row(const void* base, int is_bf16, int64_t s, int64_t cap, int D,
+              int64_t n, std::vector<double>& out) {
+  out.resize(D);
+  const int64_t off = (s * cap + n) * static_cast<int64_t>(D);
+  for (int d = 0; d < D; ++d) out[d] = widen(base, is_bf16, off + d);
+}
+
+double dot(const std::vector<double>& a, const std::vector<double>& b) {
+  double acc = 0.0;
+  for (size_t d = 0; d < a.size(); ++d) acc += a[d] * b[d];
+  return acc;
+}
+
+double l2norm(const std::vector<double>& a) { return std::sqrt(dot(a, a)); }
+
+// cos(a, b) = a.b / (max(|a|,eps) max(|b|,eps)); a zero vector gives 0.
+double cosine(const std::vector<double>& a, const std::vector<double>& b) {
+  const double eps = 1e-12;
+  return dot(a, b) / (std::max(l2norm(a), eps) * std::max(l2norm(b), eps));
+}
+
+// Strict "x ranks above y" for (score desc, index asc), NaN lowest.
+bool ranks_above(double xs, int64_t xi, double ys, int64_t yi) {
+  const bool xn = std::isnan(xs), yn = std::isnan(ys);
+  if (xn || yn) {
+    if (xn && yn) return xi < yi;
+    return yn;  // a number ranks above NaN
+  }
+  if (xs != ys) return xs > ys;
+  return xi < yi;
+}
+
+}  // namespace
+
+extern "C" {
+
+// Recent-frame count r. Appendix B.2 fixes r = 0.125 f as the default ratio;
+// rounding to an integer frame count is our reading (half rounds up), never
+// below one frame. A positive override is returned unchanged.
+int oracle_recent_frames(int64_t n_frames, int override_r) {
+  if (override_r > 0) return override_r;
+  const int64_t r = static_cast<int64_t>(std::floor(n_frames / 8.0 + 0.5));
+  return static_cast<int>(std::max<int64_t>(1, r));
+}
+
+// TaR and VaN scores for every past token of every slab (Sec. 3.1 Eq. tar,
+// Sec. 3.2). k, v: [n_slabs][cap][D]; patch_id: [n_slabs][cap] or NULL.
+// tar_out, van_out: [n_slabs][n_tokens]; entries of the r recent frames are
+// written as 0 (those tokens are always kept and are never scored).
+// Returns 0, or -1 on bad arguments (incl. a patch id >= p).
+int oracle_scores(const void* k, const void* v, int is_bf16, int64_t n_slabs,
+                  int64_t cap, int D, int64_t n_tokens, int p, int r,
+                  const uint16_t* patch_id, double* tar_out, double* van_out) {
+  if (!k || !v || !tar_out || !van_out || n_slabs < 0 || D <= 0 || p <= 0 ||
+      r <= 0 || n_tokens < 0 || n_tokens > cap || n_tokens % p != 0)
+    return -1;
+  const int64_t rp = static_cast<int64_t>(r) * p;
+  if (rp > n_tokens) return -1;
+  const int64_t n_past = n_tokens - rp;
+  std::vector<double> kp, kr, vv;
+  for (int64_t s = 0; s < n_slabs; ++s) {
+    double* tar = tar_out + s * n_tokens;
+    double* van = van_out + s * n_tokens;
+    for (int64_t n = 0; n < n_tokens; ++n) tar[n] = van[n] = 0.0;
+    for (int64_t n = 0; n < n_past; ++n) {
+      const int64_t q = patch_id ? patch_id[s * cap + n] : n % p;
+      if (q < 0 || q >= p) return -1;
+      load_row(k, is_bf16, s, cap, D, n, kp);
+      double sum_cos = 0.0;
+      for (int t = 0; t < r; ++t) {
+        load_row(k, is_bf16, s, cap, D, n_past + static_cast<int64_t>(t) * p + q, kr);
+        sum_cos += cosine(kp, kr);
+      }
+      tar[n] = -sum_cos / r;
+      load_row(v, is_bf16, s, cap, D, n, vv);
+      van[n] = l2norm(vv);
+    }
+  }
+  return 0;
+}
+
+// Budget split used by the selection (Sec. 3.3, Algorithm 1 steps 3-5):
+// out[0] = r p (recent tokens kept), out[1] = TaR picks among past tokens,
+// out[2] = VaN picks among the remaining past tokens. The pass-through case
+// (n_tokens <= budget) is reported as out = {-1,-1,-1}. Returns -1 when the
+// arguments admit no selection (r p >= budget, alpha outside [0,1] or NaN).
+int oracle_budget_split(int64_t n_tokens, int p, int r, int64_t budget,
+                        double alpha, int64_t* out) {
+  if (n_tokens <= budget) {
+    out[0] = out[1] = out[2] = -1;
+    return 0;
+  }
+  const int64_t rp = static_cast<int64_t>(r) * p;
+  if (rp >= budget || alpha < 0.0 || alpha > 1.0 || !(alpha == alpha)) return -1;
+  const int64_t tar_share = static_cast<int64_t>(std::floor(alpha * static_cast<double>(budget)));
+  const int64_t n_tar = std::max<int64_t>(0, tar_share - rp);
+  out[0] = rp;
+  out[1] = n_tar;
+  out[2] = budget - rp - n_tar;
+  return 0;
+}
+
+// Selection (Algorithm 1 steps 3-5 with the Sec. 3.3 split). tar, van:
+// [n_slabs][n_tokens] scores (recent entries ignored). kept_out:
+// [n_slabs][budget], ascending per slab; in the pass-through case
+// (n_tokens <= budget) it is 0..n_tokens-1 followed by -1.
+// gaps_out (optional, [n_slabs][2]): per stage the score gap between the last
+// token taken and the first token left, |s_(k) - s_(k+1)|; the VaN entry is
+// relative to |s_(k)|. +inf when the stage has nothing to decide.
+int oracle_select(const double* tar, const double* van, int64_t n_slabs,
+                  int64_t n_tokens, int p, int r, int64_t budget, double alpha,
+                  int32_t* kept_out, double* gaps_out) {
+  int64_t split[3];
+  if (!tar || !van || !kept_out || p <= 0 || r <= 0 || budget <= 0) return -1;
+  if (oracle_budget_split(n_tokens, p, r, budget, alpha, split) != 0) return -1;
+  const double inf = std::numeric_limits<double>::infinity();
+  for (int64_t s = 0; s < n_slabs; ++s) {
+    int32_t* kept = kept_out + s * budget;
+    if (split[0] < 0) {  // pass-through: nothing to evict
+      for (int64_t j = 0; j < budget; ++j) kept[j] = j < n_tokens ? static_cast<int32_t>(j) : -1;
+      if (gaps_out) gaps_out[2 * s] = gaps_out[2 * s + 1] = inf;
+      continue;
+    }
+    const double* ts = tar + s * n_tokens;
+    const double* vs = van + s * n_tokens;
+    const int64_t rp = split[0], n_tar = split[1], n_van = split[2];
+    const int64_t n_past = n_tokens - rp;
+
+    // TaR stage: order past tokens by (s_TaR desc, index asc).
+    std::vector<int64_t> past(n_past);
+    for (int64_t n = 0; n < n_past; ++n) past[n] = n;
+    std::vector<int64_t> by_tar = past;
+    std::sort(by_tar.begin(), by_tar.end(), [&](int64_t a, int64_t b) {
+      return ranks_above(ts[a], a, ts[b], b);
+    });
+    std::vector<char> keep(n_tokens, 0);
+    for (int64_t n = n_past; n < n_tokens; ++n) keep[n] = 1;  // recent frames
+    for (int64_t i = 0; i < n_tar; ++i) keep[by_tar[i]] = 1;
+    double gap_tar = inf;
+    if (n_tar > 0 && n_tar < n_past)
+      gap_tar = std::fabs(ts[by_tar[n_tar - 1]] - ts[by_tar[n_tar]]);
+
+    // VaN stage: among past tokens TaR did not take, (s_VaN desc, index asc).
+    std::vector<int64_t> rest;
+    for (int64_t n = 0; n < n_past; ++n)
+      if (!keep[n]) rest.push_back(n);
+    std::sort(rest.begin(), rest.end(), [&](int64_t a, int64_t b) {
+      return ranks_above(vs[a], a, vs[b], b);
+    });
+    for (int64_t i = 0; i < n_van; ++i) keep[rest[i]] = 1;
+    double gap_van = inf;
+    const int64_t n_rest = static_cast<int64_t>(rest.size());
+    if (n_van > 0 && n_van < n_rest) {
+      const double a = vs[rest[n_van - 1]], b = vs[rest[n_van]];
+      gap_van = std::fabs(a - b) / std::max(std::fabs(a), 1e-300);
+    }
+
+    int64_t j = 0;
+    for (int64_t n = 0; n < n_tokens; ++n)
+      if (keep[n]) kept[j++] = static_cast<int32_t>(n);
+    if (j != budget) return -2;  // cannot happen: the split sums to budget
+    if (gaps_out) {
+      gaps_out[2 * s] = gap_tar;
+      gaps_out[2 * s + 1] = gap_van;
+    }
+  }
+  return 0;
+}
+
+// Compaction (Sec. 3.1; Algorithm 2 last step): dst[s][j] = src[s][kept[s][j]]
+// row by row, bytes copied unchanged. Rows with kept == -1 are left untouched.
+int oracle_gather_rows(const void* src, void* dst, int64_t row_bytes,
+                       int64_t n_slabs, int64_t cap_src, int64_t cap_dst,
+                       const int32_t* kept, int64_t budget) {
+  if (!src || !dst || !kept || row_bytes <= 0) return -1;
+  const char* s8 = static_cast<const char*>(src);
+  char* d8 = static_cast<char*>(dst);
+  for (int64_t s = 0; s < n_slabs; ++s)
+    for (int64_t j = 0; j < budget; ++j) {
+      const int32_t n = kept[s * budget + j];
+      if (n < 0) continue;
+      if (n >= cap_src || j >= cap_dst) return -1;
+      std::memcpy(d8 + (s * cap_dst + j) * row_bytes, s8 + (s * cap_src + n) * row_bytes,
+                  static_cast<size_t>(row_bytes));
+    }
+  return 0;
+}
+
+// Patch ids travel with their tokens: dst[s][j] = src ? src[s][kept] : kept mod p.
+int oracle_gather_patch(const uint16_t* src_pid, uint16_t* dst_pid, int64_t n_slabs,
+                        int64_t cap_src, int64_t cap_dst, int p,
+                        const int32_t* kept, int64_t budget) {
+  if (!dst_pid || !kept || p <= 0) return -1;
+  for (int64_t s = 0; s < n_slabs; ++s)
+    for (int64_t j = 0; j < budget; ++j) {
+      const int32_t n = kept[s * budget + j];
+      if (n < 0) continue;
+      dst_pid[s * cap_dst + j] =
+          src_pid ? src_pid[s * cap_src + n] : static_cast<uint16_t>(n % p);
+    }
+  return 0;
+}
+
+// One whole pass over slabs [0, n_slabs): scores, selection, compaction of K
+// and V (and of patch ids when dst_pid != NULL). Used to time the oracle.
+int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
+                    int64_t cap, int D, int64_t n_tokens, int p, int r,
+                    int64_t budget, double alpha, const uint16_t* src_pid,
+                    void* k_dst, void* v_dst, uint16_t* dst_pid, int32_t* kept_out) {
+  std::vector<double> tar(static_cast<size_t>(n_slabs * n_tokens));
+  std::vector<double> van(tar.size());
+  if (n_tokens > budget) {
+    if (oracle_scores(k, v, is_bf16, n_slabs, cap, D, n_tokens, p, r, src_pid,
+                      tar.data(), van.data()) != 0)
+      return -1;
+  }
+  if (oracle_select(tar.data(), van.data(), n_slabs, n_tokens, p, r, budget, alpha,
+                    kept_out, nullptr) != 0)
+    return -1;
+  if (n_tokens <= budget) return 0;  // pass-through leaves the cache as it is
+  const int64_t row_bytes = static_cast<int64_t>(D) * (is_bf16 ? 2 : 4);
+  if (oracle_gather_rows(k, k_dst, row_bytes, n_slabs, cap, cap, kept_out, budget) != 0) return -1;
+  if (oracle_gather_rows(v, v_dst, row_bytes, n_slabs, cap, cap, kept_out, budget) != 0) return -1;
+  if (dst_pid &&
+      oracle_gather_patch(src_pid, dst_pid, n_slabs, cap, cap, p, kept_out, budget) != 0)
+    return -1;
+  return 0;
+}
+
+}  // extern "C"

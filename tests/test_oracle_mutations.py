@@ -1,0 +1,74 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each case plants one mistake (a flipped sign, a dropped term, a wrong index,
+a wrong tie-break, ...) in a copy of oracle/ipv_oracle.cpp, builds the copy on
+the CPU, and runs the pin suite (test_oracle_pins.py) against it. Every
+mutant must make that suite fail; the unmutated copy must pass it.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+import oracle
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "ipv_oracle.cpp")
+
+MUTANTS = [
+    ("TaR sign dropped", "tar[n] = -sum_cos / r;", "tar[n] = sum_cos / r;"),
+    ("TaR 1/r dropped", "tar[n] = -sum_cos / r;", "tar[n] = -sum_cos;"),
+    ("recent row ignores the patch",
+     "n_past + static_cast<int64_t>(t) * p + q", "n_past + static_cast<int64_t>(t) * p"),
+    ("recent rows shifted one frame back",
+     "n_past + static_cast<int64_t>(t) * p + q", "n_past - p + static_cast<int64_t>(t) * p + q"),
+    ("cosine misses the past-key norm",
+     "std::max(l2norm(a), eps) * std::max(l2norm(b), eps)", "std::max(l2norm(b), eps)"),
+    ("VaN squared norm", "van[n] = l2norm(vv);", "van[n] = dot(vv, vv);"),
+    ("VaN scored on keys", "load_row(v, is_bf16, s, cap, D, n, vv);",
+     "load_row(k, is_bf16, s, cap, D, n, vv);"),
+    ("ties go to the higher index", "  return xi < yi;\n}\n\n}  // namespace",
+     "  return xi > yi;\n}\n\n}  // namespace"),
+    ("lower score wins", "if (xs != ys) return xs > ys;", "if (xs != ys) return xs < ys;"),
+    ("alpha|C| rounded up", "std::floor(alpha * ", "std::ceil(alpha * "),
+    ("recent frames outside the TaR share", "tar_share - rp)", "tar_share)"),
+    ("patch ids ignored", "patch_id ? patch_id[s * cap + n] : n % p", "n % p"),
+    ("VaN stage may retake TaR picks", "if (!keep[n]) rest.push_back(n);", "rest.push_back(n);"),
+    ("gather copies the wrong row", "s8 + (s * cap_src + n) * row_bytes",
+     "s8 + (s * cap_src + j) * row_bytes"),
+    ("bf16 widened with the wrong shift", "<< 16;", "<< 15;"),
+    ("default r not rounded", "n_frames / 8.0 + 0.5", "n_frames / 8.0"),
+    ("recent tokens not kept", "for (int64_t n = n_past; n < n_tokens; ++n) keep[n] = 1;",
+     "for (int64_t n = n_past; n + 1 < n_tokens; ++n) keep[n] = 1;"),
+]
+
+
+def _run_pins_with(lib_path: str) -> int:
+    env = dict(os.environ, IPV_ORACLE_LIB_OVERRIDE=lib_path)
+    cmd = [sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+           os.path.join(ROOT, "tests", "test_oracle_pins.py")]
+    return subprocess.run(cmd, env=env, cwd=ROOT, capture_output=True, timeout=300).returncode
+
+
+def _build_variant(tmp_path, name: str, text: str) -> str:
+    src = tmp_path / f"{name}.cpp"
+    src.write_text(text)
+    out = str(tmp_path / f"lib{name}.so")
+    subprocess.run(oracle.build_cmd(str(src), out), check=True)
+    return out
+
+
+def test_unmutated_copy_passes(tmp_path):
+    with open(SRC) as fh:
+        text = fh.read()
+    assert _run_pins_with(_build_variant(tmp_path, "clean", text)) == 0
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_mutant_is_caught(tmp_path, name, old, new):
+    with open(SRC) as fh:
+        text = fh.read()
+    assert text.count(old) == 1, f"mutation anchor not unique/present: {old!r}"
+    lib = _build_variant(tmp_path, "mutant", text.replace(old, new))
+    assert _run_pins_with(lib) != 0, f"pins did not catch: {name}"
