@@ -1,0 +1,392 @@
+#!/usr/bin/env python3
+"""Benchmark of the InfiniPot-V compression pass on GB300.
+
+`python bench.py [--gpus N] [--steps K] [--warmup W] [--config llava]`
+prints one JSON line. A step is one whole compression pass (recent-frame
+mean, TaR/VaN scoring, split-budget selection, compaction) over every
+(layer, KV head) slab of a seeded synthetic cache already resident in HBM;
+the L2 is flushed (256 MiB write) between timed passes. Under torchrun each
+rank runs its own independent stream (weak scaling; no data-path
+collective). `--impl reference` times the CPU oracle instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "compress-pass latency (ms) and HBM GB/s vs GB300 peak, 7B shape 6K budget"
+KERNELS = ("recent_mean", "score", "select", "gather")
+FALLBACK_HBM_GBS = 6800.0
+
+
+def workload_desc(w: synth.Workload) -> str:
+    return (f"{w.name}: {w.n_streams}x{w.n_layers} layers x {w.n_kv_heads} KV heads x "
+            f"head_dim {w.head_dim} {w.dtype}, {w.grid_h}x{w.grid_w} tokens/frame, "
+            f"{w.n_frames} frames ({w.n_tokens} tokens) -> budget {w.budget}, alpha {w.tar_ratio}")
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            return float(json.load(fh)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def bytes_model(w: synth.Workload, S: int, r: int):
+    """Algorithmic bytes: the pass total of the design contract and per kernel."""
+    s, D, N, C, p = w.elem_bytes, w.head_dim, w.n_tokens, w.budget, w.p
+    rp = r * p
+    n_past = N - rp
+    row = D * s
+    pass_bytes = S * row * (2 * N + 4 * C) + S * C * 4
+    tight = S * row * (2 * N - rp + 4 * C) + S * C * 4
+    per_kernel = {
+        "recent_mean": S * (rp * row + p * D * 4),
+        "score": S * (2 * n_past * row + 8 * n_past),
+        "select": S * (8 * n_past + 4 * C),
+        "gather": S * (4 * C * row + 4 * C),
+    }
+    return pass_bytes, tight, per_kernel
+
+
+def source_digest() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2506_15745_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as fh:
+            h.update(name.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    try:
+        with open(path) as fh:
+            rec = json.load(fh)
+    except Exception:
+        return None
+    ent = rec.get("kernels", {}).get(kernel)
+    if not ent or rec.get("source_digest") != source_digest() or rec.get("workload") != workload:
+        return None
+    return ent.get("dram_bytes_per_launch_full_size")
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"],
+                    "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=10)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def time_oracle(w: synth.Workload, k_np, v_np, r: int, budget_s: float = 12.0):
+    """Oracle ms per full pass, from a bounded sample of slabs (single thread)."""
+    import oracle
+    oracle.build()
+    S_total = w.n_slabs
+    t0 = time.perf_counter()
+    oracle.compress(k_np[:1], v_np[:1], w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+    t1 = time.perf_counter() - t0
+    n = int(max(1, min(k_np.shape[0], round(budget_s / max(t1, 1e-6)))))
+    t0 = time.perf_counter()
+    oracle.compress(k_np[:n], v_np[:n], w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+    dt = time.perf_counter() - t0
+    ms_pass = dt * 1e3 * S_total / n
+    return ms_pass, n, dt
+
+
+def run_reference(args, w: synth.Workload):
+    """The reference arm: the CPU oracle as it stands, on host cores, rank 0 only."""
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    r = oracle.recent_frames(w.n_frames)
+    K1, V1 = synth.host_generate(w.scaled(n_layers=1, n_kv_heads=1, n_streams=1))
+    t0 = time.perf_counter()
+    oracle.compress(K1, V1, w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+    t_slab = time.perf_counter() - t0
+    # Slabs per step: at most --ref-slabs, fewer if the run would exceed ~2 min.
+    fit = int(120.0 / max(1e-6, (args.steps + args.warmup) * t_slab))
+    per_step_slabs = max(1, min(w.slabs_per_stream, args.ref_slabs, fit))
+    ws = w.scaled(n_layers=1, n_kv_heads=per_step_slabs, n_streams=1)
+    K, V = synth.host_generate(ws)
+    for _ in range(args.warmup):
+        oracle.compress(K[:1], V[:1], w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.compress(K, V, w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+        times.append(time.perf_counter() - t0)
+    ms = float(np.mean(times)) * 1e3 * w.n_slabs / per_step_slabs
+    sample = (f"{per_step_slabs} of {w.n_slabs} slabs per step (host-generated, same recipe), "
+              f"extrapolated x{w.n_slabs / per_step_slabs:.1f} to a full pass")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": ms, "unit": "ms", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": workload_desc(w)},
+        "cpu_baseline": {"value": ms, "unit": "ms", "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": ms, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args, w: synth.Workload):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2506_15745_gb300 import ipv
+    from paper_2506_15745_gb300.cache import PingPongCache
+    from paper_2506_15745_gb300.shard import max_over_ranks, shard_range
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    # Units of work on this rank: whole streams. Single-stream configs run one
+    # independent replica stream per rank; multi-stream configs are sharded.
+    if w.n_streams > 1:
+        s0, s1 = shard_range(w.n_streams, rank, world)
+        streams = list(range(s0, s1))
+    else:
+        streams = [rank]
+    per = w.slabs_per_stream
+    S = per * len(streams)
+    N, C, D, p = w.n_tokens, w.budget, w.head_dim, w.p
+
+    ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
+             token_capacity=N)
+    r = ipv.recent_frames(w.n_frames)
+    cache = PingPongCache(S, N, D, w.dtype, patch_ids=False)
+    for i, st in enumerate(streams):
+        synth.device_generate(w, cache.k[0, i * per:(i + 1) * per], cache.v[0, i * per:(i + 1) * per],
+                              stream=st)
+    kept = torch.empty((S, C), dtype=torch.int32, device="cuda")
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    L = len(streams) * w.n_layers
+
+    def one_pass():
+        k, v = cache.structs(pid_valid=False)
+        k.cur = v.cur = 0
+        ipv.compress(k, v, L, w.n_kv_heads, D, N, w.grid_h, w.grid_w, C, w.tar_ratio, kept)
+
+    for _ in range(max(3, args.warmup)):
+        flush.zero_()
+        one_pass()
+    torch.cuda.synchronize()
+
+    n_ev = args.steps
+    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(n_ev)]
+    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(n_ev)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)  # let the sampler start before the timed region
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ipv.profile_enable(True)
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()
+        ev0[i].record()
+        one_pass()
+        ev1[i].record()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter() - t_wall
+    if world > 1:
+        dist.barrier()
+    ipv.profile_enable(False)
+    clk = clocks.stop()
+    prof = ipv.profile_collect()
+    per_pass = np.array([a.elapsed_time(b) for a, b in zip(ev0, ev1)])
+    ms_pass = float(per_pass.mean())
+    ms_pass_max = max_over_ranks(ms_pass)
+    wall_max = max_over_ranks(t_wall)
+
+    pass_bytes, tight_bytes, kbytes = bytes_model(w, S, r)
+    peak, peak_kind = peaks()
+    kern_ms = {k: (prof[k][0] / prof[k][1] if prof[k][1] else 0.0) for k in KERNELS}
+    dominant = max(KERNELS, key=lambda k: prof[k][0])
+    achieved = kbytes[dominant] / (kern_ms[dominant] * 1e-3) / 1e9
+    traffic = ncu_traffic(dominant, w.name) if S == w.slabs_per_stream else None
+    launches = sum(prof[k][1] for k in KERNELS)
+
+    # End to end through the public API with host buffers: pinned H2D of the
+    # step's K and V, the pass, D2H of the kept indices and compacted rows.
+    e2e_steps = max(3, min(args.e2e_steps, args.steps))
+    k_host = torch.empty((S, N, D), dtype=cache.k.dtype, pin_memory=True)
+    v_host = torch.empty_like(k_host, pin_memory=True)
+    k_host.copy_(cache.k[0])
+    v_host.copy_(cache.v[0])
+    kept_host = torch.empty((S, C), dtype=torch.int32, pin_memory=True)
+    k_out = torch.empty((S, C, D), dtype=cache.k.dtype, pin_memory=True)
+    v_out = torch.empty_like(k_out, pin_memory=True)
+
+    def e2e_step():
+        cache.k[0].copy_(k_host, non_blocking=True)
+        cache.v[0].copy_(v_host, non_blocking=True)
+        one_pass()
+        kept_host.copy_(kept, non_blocking=True)
+        k_out.copy_(cache.k[1, :, :C], non_blocking=True)
+        v_out.copy_(cache.v[1, :, :C], non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+    for i in range(e2e_steps):
+        flush.zero_()
+        e0[i].record()
+        e2e_step()
+        e1[i].record()
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(float(np.mean([a.elapsed_time(b) for a, b in zip(e0, e1)])))
+    h2d = 2 * k_host.numel() * k_host.element_size()
+    d2h = kept_host.numel() * 4 + 2 * k_out.numel() * k_out.element_size()
+
+    line = None
+    if rank == 0:
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            n_s = min(S, 128)
+            k_np = cache.k[0, :n_s].contiguous()
+            v_np = cache.v[0, :n_s].contiguous()
+            if w.is_bf16:
+                k_np = k_np.view(torch.int16).cpu().numpy().view(np.uint16)
+                v_np = v_np.view(torch.int16).cpu().numpy().view(np.uint16)
+            else:
+                k_np, v_np = k_np.cpu().numpy(), v_np.cpu().numpy()
+            wc = w.scaled(n_streams=len(streams))
+            ms_cpu, n_used, secs = time_oracle(wc, k_np, v_np, r, args.cpu_seconds)
+            cpu = {"value": ms_cpu, "unit": "ms", "cores": 1, "kind": "oracle",
+                   "sample": f"{n_used} of {S} slabs of this workload ({secs:.1f} s, single "
+                             f"thread), extrapolated x{S / n_used:.1f} to a full pass",
+                   "host_cores_available": len(os.sched_getaffinity(0))}
+        tokens_scored = world * S * N / (ms_pass_max * 1e-3)
+        line = {
+            "metric": METRIC, "value": ms_pass_max, "unit": "ms", "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_pass_max,
+            "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": workload_desc(w), "storage_dtype": w.dtype,
+                       "streams_per_gpu": len(streams), "slabs_per_gpu": S,
+                       "recent_frames": r,
+                       "l2": "flushed (256 MiB write) before every timed pass; inputs "
+                             f"{2 * S * N * D * w.elem_bytes / 1e6:.0f} MB > L2",
+                       "parallelism": f"independent streams, {world} GPU(s), no collective"},
+            "pass_bytes": pass_bytes,
+            "pass_gbs": pass_bytes / (ms_pass_max * 1e-3) / 1e9,
+            "pass_roofline_frac": pass_bytes / (ms_pass_max * 1e-3) / 1e9 / peak,
+            "pass_bytes_tight": tight_bytes,
+            "tokens_scored_per_s": tokens_scored,
+            "per_pass_ms_p50": float(np.percentile(per_pass, 50)),
+            "per_pass_ms_p99": float(np.percentile(per_pass, 99)),
+            "kernel_ms": {k: round(kern_ms[k], 5) for k in KERNELS},
+            "roofline": {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": peak,
+                         "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)" if peak_kind == "measured" else "fallback 6.8 TB/s",
+                         "unit": "GB/s", "frac": achieved / peak, "traffic": traffic,
+                         "algorithmic_bytes": kbytes[dominant]},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_ms, "unit": "ms", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+            "gpu_launches": launches,
+            "timed_wall_s": wall_max,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    ipv.shutdown()
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return line
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--config", default="llava", choices=sorted(synth.CONFIGS))
+    ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ref-slabs", type=int, default=4)
+    args = ap.parse_args(argv)
+    w = synth.CONFIGS[args.config]
+    if args.config == "stream":
+        w = w.scaled(name="stream")
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_gpu(args, w)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,163 @@
+/*
+ * ipv.h -- C ABI of the GB300 (sm_103a) InfiniPot-V KV-cache compression pass.
+ *
+ * InfiniPot-V (arXiv 2506.15745) keeps a streaming video MLLM's KV cache under
+ * a fixed memory cap |M|: whenever the cache reaches |M| tokens it is cut to a
+ * target size |C| (Algorithm 1). For every (layer, KV head) "slab" the pass
+ *   (i)   scores each past vision token with Temporal-axis Redundancy
+ *         s_TaR = -(1/r) sum_{t'} cos(K_past[t,i,j], K_recent[t',i,j])
+ *         (Sec. 3.1, Eq. tar; the cache is viewed as f frames of p patches,
+ *         the r latest frames are "recent");
+ *   (ii)  scores it with Value Norm s_VaN = ||V[t,i,j]||_2 (Sec. 3.2);
+ *   (iii) keeps the r*p recent tokens, then the floor(alpha |C|) - r*p past
+ *         tokens of highest s_TaR, then fills the rest of |C| with the past
+ *         tokens of highest s_VaN that TaR did not take (Sec. 3.3, Algorithm 1
+ *         steps 3-5; Algorithm 2's max-forcing of TaR picks before its final
+ *         TopK); ties go to the lower token index, NaN ranks lowest;
+ *   (iv)  compacts K and V to the kept rows in ascending index order
+ *         (Sec. 3.1, K~ = K[:, I, :]; Algorithm 2 last step).
+ *
+ * Memory layout (all device memory, owned by the caller unless stated):
+ *   K or V cache half : [n_layers][n_kv_heads][token_capacity][head_dim],
+ *                       contiguous, element type chosen in ipv_init (bf16 or
+ *                       fp32), 16-byte aligned; row n of slab s starts at
+ *                       element (s * token_capacity + n) * head_dim.
+ *   patch ids         : uint16 [n_layers][n_kv_heads][token_capacity]: the
+ *                       frame-grid position (i*w + j) of each cached token.
+ *   scores            : fp32 [n_slabs][n_tokens].
+ *   kept indices      : int32 [n_slabs][budget], ascending per slab.
+ *
+ * Frames: the n_tokens rows of a slab hold f = n_tokens / p frames' worth of
+ * tokens (p = frame_grid_h * frame_grid_w). The last r*p rows are the r most
+ * recent frames, whole and in patch order. The patch of a past row n is
+ * patch_id[n] when the cache half has patch ids, else n mod p (a cache that
+ * has never been compacted).
+ *
+ * Execution: every compute entry point validates its arguments on the host,
+ * then enqueues kernels on the given CUDA stream and returns without waiting.
+ * No entry point synchronises the device or the stream, and none allocates
+ * device memory except ipv_init. The library keeps one global state (device,
+ * element type, scratch); calls are not thread-safe and must come from one
+ * host thread at a time. Errors never trap on the device.
+ */
+#ifndef IPV_H_
+#define IPV_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  IPV_OK = 0,
+  IPV_EINVAL = 1,   /* bad argument; nothing was enqueued */
+  IPV_ENOINIT = 2,  /* ipv_init has not succeeded (or ipv_shutdown was called) */
+  IPV_ENOMEM = 3,   /* device allocation failed in ipv_init */
+  IPV_ECUDA = 4,    /* CUDA runtime error; see ipv_last_error() */
+  IPV_ETIMEOUT = 5  /* a bounded host wait ran out (profiling read-back only) */
+} ipv_status;
+
+typedef enum { IPV_BF16 = 0, IPV_F32 = 1 } ipv_dtype;
+
+typedef struct {
+  int device;             /* CUDA device ordinal */
+  ipv_dtype dtype;        /* element type of K and V */
+  int recent_frames;      /* r; 0 = max(1, floor(f/8 + 1/2)), the r = 0.125 f
+                             default of Appendix B.2 */
+  int max_head_dim;       /* largest head_dim any call will use (<= 512) */
+  int max_frame_tokens;   /* largest p = frame_grid_h*frame_grid_w (<= 65535) */
+  int64_t max_slabs;      /* largest n_layers*n_kv_heads any call will use */
+  int64_t token_capacity; /* rows per slab in each cache half (the slab stride) */
+} ipv_options;
+
+/* One tensor (K or V) of the ping-pong cache: two halves of identical
+ * layout; buf[cur] holds the live rows. patch_id[h] may be NULL. */
+typedef struct {
+  void* buf[2];
+  uint16_t* patch_id[2];
+  int cur;
+} ipv_kv;
+
+/* Largest n_tokens the selection kernel accepts (its keys live in shared memory). */
+#define IPV_MAX_TOKENS 49152
+
+/* Initialise the library on opt->device: checks the device, allocates the
+ * scratch (per-token scores and per-patch recent-frame means, sized from
+ * max_slabs, token_capacity, max_frame_tokens and max_head_dim). Calling it
+ * again first releases the previous state. Errors: IPV_EINVAL (bad options),
+ * IPV_ECUDA (no usable device), IPV_ENOMEM. */
+ipv_status ipv_init(const ipv_options* opt);
+
+/* Release the scratch and forget the options. Waits for the device first. */
+void ipv_shutdown(void);
+
+/* The compression pass, steps (i)-(iv) above, for every (layer, KV head) slab.
+ *   k, v          : caches; rows 0..n_tokens-1 of buf[cur] are read, the
+ *                   budget survivors are written to rows 0..budget-1 of
+ *                   buf[1-cur] and cur is flipped (host-side) in both structs.
+ *                   Patch ids: read from k->patch_id[k->cur] (NULL: n mod p);
+ *                   written to k->patch_id[1-k->cur] if it is not NULL.
+ *                   v->patch_id is not used.
+ *   n_tokens      : |M|, rows currently cached per slab; multiple of p.
+ *   budget        : |C|, rows kept per slab; r*p < budget.
+ *   tar_ratio     : alpha in [0, 1]; the TaR share is floor(alpha * budget).
+ *   kept_idx_out  : device int32 [n_layers*n_kv_heads][budget]: the kept
+ *                   source rows, ascending per slab.
+ *   stream        : a cudaStream_t (NULL = legacy default stream).
+ * Pass-through: if n_tokens <= budget nothing is evicted: kept_idx_out gets
+ * 0..n_tokens-1 then -1 padding, no row is copied and cur is not flipped.
+ * Errors: IPV_EINVAL (checked before anything is enqueued: non-positive
+ * sizes, n_tokens not a multiple of p or above token_capacity or
+ * IPV_MAX_TOKENS, budget above token_capacity, tar_ratio outside [0,1] or NaN,
+ * r*p >= budget, head_dim*elem_size not a multiple of 16 bytes, sizes above
+ * the ipv_init maxima, NULL or misaligned pointers, the two halves aliasing),
+ * IPV_ENOINIT, IPV_ECUDA (launch failure). */
+ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int head_dim,
+                        int64_t n_tokens, int frame_grid_h, int frame_grid_w, int64_t budget,
+                        float tar_ratio, int32_t* kept_idx_out, void* stream);
+
+/* Steps (i) and (ii) only, for inspection and parity checks: fp32 s_TaR and
+ * s_VaN of every token of every slab into tar_out / van_out (device,
+ * [n_slabs][n_tokens]). Entries of the r recent frames are written as 0.
+ * Requires n_tokens > r*p. Same argument rules as ipv_compress (budget and
+ * tar_ratio aside); the caches are only read. */
+ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_heads,
+                     int head_dim, int64_t n_tokens, int frame_grid_h, int frame_grid_w,
+                     float* tar_out, float* van_out, void* stream);
+
+/* Step (iii) only: the split-budget selection on given fp32 scores (device,
+ * [n_slabs][n_tokens]; entries of the recent frames are ignored), writing
+ * kept_idx_out as ipv_compress does. Pass-through and errors as ipv_compress. */
+ipv_status ipv_select(const float* tar, const float* van, int64_t n_slabs, int64_t n_tokens,
+                      int frame_grid_h, int frame_grid_w, int64_t budget, float tar_ratio,
+                      int32_t* kept_idx_out, void* stream);
+
+/* The recent-frame count r the library uses for a cache of n_frames frames
+ * (the ipv_init override if set, else max(1, floor(n_frames/8 + 1/2))).
+ * Returns -1 before ipv_init. */
+int ipv_recent_frames(int64_t n_frames);
+
+/* Message of the last failed call on this thread ("" if none). */
+const char* ipv_last_error(void);
+
+/* Static name of a status code. */
+const char* ipv_status_string(ipv_status s);
+
+/* Kernel timing for benchmarks: while enabled, ipv_compress and ipv_score
+ * record CUDA events around each kernel on the call's stream. Kernel ids:
+ * 0 recent-frame mean, 1 scoring, 2 selection, 3 compaction. */
+#define IPV_NUM_KERNELS 4
+ipv_status ipv_profile_enable(int on);
+
+/* Waits (at most timeout_ms) for the recorded events, then writes per kernel
+ * id the summed device time in ms and the number of launches, and clears the
+ * record. Errors: IPV_ETIMEOUT, IPV_ECUDA, IPV_EINVAL (NULL outputs). */
+ipv_status ipv_profile_collect(double ms_out[IPV_NUM_KERNELS],
+                               int64_t launches_out[IPV_NUM_KERNELS], int timeout_ms);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* IPV_H_ */

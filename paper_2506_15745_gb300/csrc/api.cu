@@ -1,0 +1,466 @@
+// C ABI of libipv.so (declared in include/ipv.h): state, argument checks,
+// kernel sequencing and optional per-kernel event timing.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <ctime>
+#include <string>
+#include <vector>
+
+#include "ipv.h"
+#include "ipv_common.cuh"
+
+namespace {
+
+struct EventPair {
+  cudaEvent_t start = nullptr, stop = nullptr;
+};
+
+struct State {
+  bool ready = false;
+  ipv_options opt{};
+  int num_sms = 0;
+  float* tar = nullptr;   // [max_slabs][token_capacity]
+  float* van = nullptr;
+  float* m = nullptr;     // [max_slabs][max_frame_tokens][max_head_dim]
+  bool profiling = false;
+  std::vector<EventPair> pool;                      // idle event pairs
+  std::vector<EventPair> pending[IPV_NUM_KERNELS];  // recorded, not yet read
+};
+
+State g;
+thread_local std::string g_err;
+
+ipv_status fail(ipv_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = std::string(ipv_status_string(s)) + ": " + buf;
+  return s;
+}
+
+ipv_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(IPV_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int elem_bytes() { return g.opt.dtype == IPV_BF16 ? 2 : 4; }
+
+int default_recent_frames(int64_t f) {
+  if (g.opt.recent_frames > 0) return g.opt.recent_frames;
+  const int64_t r = static_cast<int64_t>(std::floor(static_cast<double>(f) / 8.0 + 0.5));
+  return static_cast<int>(r < 1 ? 1 : r);
+}
+
+// ------------------------------------------------------------------ profiling
+EventPair take_pair() {
+  if (!g.pool.empty()) {
+    EventPair p = g.pool.back();
+    g.pool.pop_back();
+    return p;
+  }
+  EventPair p;
+  cudaEventCreate(&p.start);
+  cudaEventCreate(&p.stop);
+  return p;
+}
+
+void prof_begin(int id, cudaStream_t st) {
+  if (!g.profiling) return;
+  EventPair p = take_pair();
+  cudaEventRecord(p.start, st);
+  g.pending[id].push_back(p);
+}
+
+void prof_end(int id, cudaStream_t st) {
+  if (!g.profiling || g.pending[id].empty()) return;
+  cudaEventRecord(g.pending[id].back().stop, st);
+}
+
+void release_events() {
+  for (auto& v : g.pending) {
+    for (auto& p : v) g.pool.push_back(p);
+    v.clear();
+  }
+  for (auto& p : g.pool) {
+    cudaEventDestroy(p.start);
+    cudaEventDestroy(p.stop);
+  }
+  g.pool.clear();
+}
+
+// ------------------------------------------------------------- argument checks
+struct Shape {
+  int64_t S, N, f;
+  int D, p, r;
+  int64_t rp;
+};
+
+// Checks that need no library state; then the init check; then the rest.
+ipv_status check_cache(const ipv_kv* k, const ipv_kv* v, int L, int H, int D, int64_t N, int gh,
+                       int gw, bool need_dst, Shape* sh) {
+  if (!k || !v) return fail(IPV_EINVAL, "k and v must not be NULL");
+  if (k->cur != 0 && k->cur != 1) return fail(IPV_EINVAL, "k->cur must be 0 or 1");
+  if (v->cur != 0 && v->cur != 1) return fail(IPV_EINVAL, "v->cur must be 0 or 1");
+  if (L <= 0 || H <= 0 || D <= 0 || N <= 0 || gh <= 0 || gw <= 0)
+    return fail(IPV_EINVAL, "sizes must be positive (layers %d heads %d head_dim %d tokens %lld grid %dx%d)",
+                L, H, D, static_cast<long long>(N), gh, gw);
+  const int64_t p = static_cast<int64_t>(gh) * gw;
+  if (p > 65535) return fail(IPV_EINVAL, "frame_grid_h*frame_grid_w = %lld exceeds 65535", static_cast<long long>(p));
+  if (N % p != 0)
+    return fail(IPV_EINVAL, "n_tokens %lld is not a multiple of the %lld tokens of a frame",
+                static_cast<long long>(N), static_cast<long long>(p));
+  const void* src_k = k->buf[k->cur];
+  const void* src_v = v->buf[v->cur];
+  if (!src_k || !src_v) return fail(IPV_EINVAL, "live cache halves buf[cur] must not be NULL");
+  if (!aligned16(src_k) || !aligned16(src_v)) return fail(IPV_EINVAL, "cache halves must be 16-byte aligned");
+  if (src_k == src_v) return fail(IPV_EINVAL, "k and v share one buffer");
+  if (need_dst) {
+    const void* dk = k->buf[1 - k->cur];
+    const void* dv = v->buf[1 - v->cur];
+    if (!dk || !dv) return fail(IPV_EINVAL, "destination halves buf[1-cur] must not be NULL");
+    if (!aligned16(dk) || !aligned16(dv)) return fail(IPV_EINVAL, "cache halves must be 16-byte aligned");
+    if (dk == src_k || dv == src_v || dk == src_v || dv == src_k || dk == dv)
+      return fail(IPV_EINVAL, "ping-pong halves must be distinct buffers");
+    const uint16_t* ps = k->patch_id[k->cur];
+    const uint16_t* pd = k->patch_id[1 - k->cur];
+    if (pd && pd == ps) return fail(IPV_EINVAL, "patch-id halves must be distinct buffers");
+  }
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  const int64_t S = static_cast<int64_t>(L) * H;
+  if (S > g.opt.max_slabs)
+    return fail(IPV_EINVAL, "n_layers*n_kv_heads = %lld exceeds max_slabs %lld", static_cast<long long>(S),
+                static_cast<long long>(g.opt.max_slabs));
+  if (D > g.opt.max_head_dim) return fail(IPV_EINVAL, "head_dim %d exceeds max_head_dim %d", D, g.opt.max_head_dim);
+  if ((static_cast<int64_t>(D) * elem_bytes()) % 16 != 0)
+    return fail(IPV_EINVAL, "head_dim*element size must be a multiple of 16 bytes");
+  if (p > g.opt.max_frame_tokens)
+    return fail(IPV_EINVAL, "frame tokens %lld exceed max_frame_tokens %d", static_cast<long long>(p),
+                g.opt.max_frame_tokens);
+  if (N > g.opt.token_capacity)
+    return fail(IPV_EINVAL, "n_tokens %lld exceeds token_capacity %lld", static_cast<long long>(N),
+                static_cast<long long>(g.opt.token_capacity));
+  sh->S = S;
+  sh->N = N;
+  sh->D = D;
+  sh->p = static_cast<int>(p);
+  sh->f = N / p;
+  sh->r = default_recent_frames(sh->f);
+  sh->rp = static_cast<int64_t>(sh->r) * p;
+  return IPV_OK;
+}
+
+// Budget split of Sec. 3.3 / Algorithm 1: floor(alpha C) for TaR including the
+// r p recent tokens, the rest of C for VaN.
+void split_budget(int64_t budget, float tar_ratio, int64_t rp, int64_t* n_tar, int64_t* n_van) {
+  const int64_t share = static_cast<int64_t>(std::floor(static_cast<double>(tar_ratio) * budget));
+  *n_tar = share > rp ? share - rp : 0;
+  *n_van = budget - rp - *n_tar;
+}
+
+ipv_status check_select_args(int64_t N, int64_t budget, float tar_ratio, const int32_t* kept) {
+  if (!kept) return fail(IPV_EINVAL, "kept_idx_out must not be NULL");
+  if ((reinterpret_cast<uintptr_t>(kept) & 3u) != 0) return fail(IPV_EINVAL, "kept_idx_out must be 4-byte aligned");
+  if (budget <= 0) return fail(IPV_EINVAL, "budget must be positive");
+  if (!(tar_ratio >= 0.0f && tar_ratio <= 1.0f)) return fail(IPV_EINVAL, "tar_ratio must lie in [0, 1]");
+  if (budget > INT32_MAX || N > INT32_MAX) return fail(IPV_EINVAL, "sizes exceed int32 indices");
+  return IPV_OK;
+}
+
+ipv_status after_launch(cudaError_t e, const char* what) {
+  return e == cudaSuccess ? IPV_OK : cuda_fail(e, what);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ipv_status_string(ipv_status s) {
+  switch (s) {
+    case IPV_OK: return "IPV_OK";
+    case IPV_EINVAL: return "IPV_EINVAL";
+    case IPV_ENOINIT: return "IPV_ENOINIT";
+    case IPV_ENOMEM: return "IPV_ENOMEM";
+    case IPV_ECUDA: return "IPV_ECUDA";
+    case IPV_ETIMEOUT: return "IPV_ETIMEOUT";
+  }
+  return "IPV_UNKNOWN";
+}
+
+const char* ipv_last_error(void) { return g_err.c_str(); }
+
+void ipv_shutdown(void) {
+  if (!g.ready) return;
+  cudaSetDevice(g.opt.device);
+  cudaDeviceSynchronize();
+  release_events();
+  cudaFree(g.tar);
+  cudaFree(g.van);
+  cudaFree(g.m);
+  g = State{};
+}
+
+ipv_status ipv_init(const ipv_options* opt) {
+  if (!opt) return fail(IPV_EINVAL, "options must not be NULL");
+  if (opt->dtype != IPV_BF16 && opt->dtype != IPV_F32) return fail(IPV_EINVAL, "unknown dtype %d", opt->dtype);
+  if (opt->device < 0) return fail(IPV_EINVAL, "device must be >= 0");
+  if (opt->recent_frames < 0) return fail(IPV_EINVAL, "recent_frames must be >= 0");
+  if (opt->max_head_dim <= 0 || opt->max_head_dim > 512) return fail(IPV_EINVAL, "max_head_dim must be in [1, 512]");
+  if (opt->max_frame_tokens <= 0 || opt->max_frame_tokens > 65535)
+    return fail(IPV_EINVAL, "max_frame_tokens must be in [1, 65535]");
+  if (opt->max_slabs <= 0 || opt->max_slabs > INT32_MAX) return fail(IPV_EINVAL, "max_slabs must be in [1, 2^31)");
+  if (opt->token_capacity <= 0 || opt->token_capacity > INT32_MAX)
+    return fail(IPV_EINVAL, "token_capacity must be in [1, 2^31)");
+  ipv_shutdown();
+  int n_dev = 0;
+  cudaError_t e = cudaGetDeviceCount(&n_dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceCount");
+  if (opt->device >= n_dev) return fail(IPV_EINVAL, "device %d not present (%d devices)", opt->device, n_dev);
+  if ((e = cudaSetDevice(opt->device)) != cudaSuccess) return cuda_fail(e, "cudaSetDevice");
+  cudaDeviceProp prop;
+  if ((e = cudaGetDeviceProperties(&prop, opt->device)) != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
+  // Kernel images exist only for sm_103a; setting attributes fails otherwise.
+  if ((e = ipv::score_prepare(opt->max_frame_tokens, opt->max_head_dim)) != cudaSuccess)
+    return cuda_fail(e, "no usable kernel image for this device (built for sm_103a)");
+  if ((e = ipv::select_prepare(IPV_MAX_TOKENS)) != cudaSuccess) return cuda_fail(e, "select kernel set-up");
+  State s;
+  s.opt = *opt;
+  s.num_sms = prop.multiProcessorCount;
+  const size_t score_bytes = static_cast<size_t>(opt->max_slabs) * opt->token_capacity * sizeof(float);
+  const size_t m_bytes =
+      static_cast<size_t>(opt->max_slabs) * opt->max_frame_tokens * opt->max_head_dim * sizeof(float);
+  if (cudaMalloc(&s.tar, score_bytes) != cudaSuccess || cudaMalloc(&s.van, score_bytes) != cudaSuccess ||
+      cudaMalloc(&s.m, m_bytes) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(s.tar);
+    cudaFree(s.van);
+    cudaFree(s.m);
+    return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated", 2 * score_bytes + m_bytes);
+  }
+  s.ready = true;
+  g = s;
+  g_err.clear();
+  return IPV_OK;
+}
+
+int ipv_recent_frames(int64_t n_frames) {
+  if (!g.ready || n_frames <= 0) return -1;
+  return default_recent_frames(n_frames);
+}
+
+ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_heads, int head_dim,
+                     int64_t n_tokens, int frame_grid_h, int frame_grid_w, float* tar_out,
+                     float* van_out, void* stream) {
+  Shape sh;
+  if (!tar_out || !van_out) return fail(IPV_EINVAL, "tar_out and van_out must not be NULL");
+  if ((reinterpret_cast<uintptr_t>(tar_out) & 3u) || (reinterpret_cast<uintptr_t>(van_out) & 3u))
+    return fail(IPV_EINVAL, "score outputs must be 4-byte aligned");
+  ipv_status s = check_cache(k, v, n_layers, n_kv_heads, head_dim, n_tokens, frame_grid_h,
+                             frame_grid_w, false, &sh);
+  if (s != IPV_OK) return s;
+  if (sh.rp >= sh.N)
+    return fail(IPV_EINVAL, "the %d recent frames leave no past tokens to score", sh.r);
+  cudaSetDevice(g.opt.device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  ipv::ScoreArgs a{};
+  a.k = k->buf[k->cur];
+  a.v = v->buf[v->cur];
+  a.patch_id = k->patch_id[k->cur];
+  a.n_slabs = sh.S;
+  a.cap = g.opt.token_capacity;
+  a.n_tokens = sh.N;
+  a.D = sh.D;
+  a.p = sh.p;
+  a.r = sh.r;
+  a.is_bf16 = g.opt.dtype == IPV_BF16;
+  a.m = g.m;
+  a.tar = tar_out;
+  a.van = van_out;
+  a.zero_recent = 1;
+  a.num_sms = g.num_sms;
+  prof_begin(0, st);
+  cudaError_t e = ipv::launch_recent_mean(a, st);
+  prof_end(0, st);
+  if (e != cudaSuccess) return cuda_fail(e, "recent-frame mean kernel");
+  prof_begin(1, st);
+  e = ipv::launch_score(a, st);
+  prof_end(1, st);
+  return after_launch(e, "scoring kernel");
+}
+
+ipv_status ipv_select(const float* tar, const float* van, int64_t n_slabs, int64_t n_tokens,
+                      int frame_grid_h, int frame_grid_w, int64_t budget, float tar_ratio,
+                      int32_t* kept_idx_out, void* stream) {
+  if (!tar || !van) return fail(IPV_EINVAL, "score inputs must not be NULL");
+  if (n_slabs <= 0 || n_tokens <= 0 || frame_grid_h <= 0 || frame_grid_w <= 0)
+    return fail(IPV_EINVAL, "sizes must be positive");
+  ipv_status s = check_select_args(n_tokens, budget, tar_ratio, kept_idx_out);
+  if (s != IPV_OK) return s;
+  const int64_t p = static_cast<int64_t>(frame_grid_h) * frame_grid_w;
+  if (n_tokens % p != 0) return fail(IPV_EINVAL, "n_tokens is not a multiple of the frame size");
+  if (n_slabs > INT32_MAX) return fail(IPV_EINVAL, "too many slabs");
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  cudaSetDevice(g.opt.device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (n_tokens <= budget)
+    return after_launch(ipv::launch_passthrough(kept_idx_out, n_slabs, n_tokens, budget, st),
+                        "pass-through kernel");
+  if (n_tokens > IPV_MAX_TOKENS) return fail(IPV_EINVAL, "n_tokens exceeds IPV_MAX_TOKENS");
+  const int64_t rp = static_cast<int64_t>(default_recent_frames(n_tokens / p)) * p;
+  if (rp >= budget) return fail(IPV_EINVAL, "recent tokens r*p = %lld must be below budget", static_cast<long long>(rp));
+  ipv::SelectArgs a{};
+  a.tar = tar;
+  a.van = van;
+  a.n_slabs = n_slabs;
+  a.n_tokens = n_tokens;
+  a.rp = rp;
+  a.budget = budget;
+  split_budget(budget, tar_ratio, rp, &a.n_tar, &a.n_van);
+  a.kept = kept_idx_out;
+  prof_begin(2, st);
+  cudaError_t e = ipv::launch_select(a, st);
+  prof_end(2, st);
+  return after_launch(e, "selection kernel");
+}
+
+ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int head_dim,
+                        int64_t n_tokens, int frame_grid_h, int frame_grid_w, int64_t budget,
+                        float tar_ratio, int32_t* kept_idx_out, void* stream) {
+  ipv_status s = check_select_args(n_tokens, budget, tar_ratio, kept_idx_out);
+  if (s != IPV_OK) return s;
+  Shape sh;
+  s = check_cache(k, v, n_layers, n_kv_heads, head_dim, n_tokens, frame_grid_h, frame_grid_w,
+                  n_tokens > budget, &sh);
+  if (s != IPV_OK) return s;
+  if (budget > g.opt.token_capacity)
+    return fail(IPV_EINVAL, "budget %lld exceeds token_capacity %lld", static_cast<long long>(budget),
+                static_cast<long long>(g.opt.token_capacity));
+  cudaSetDevice(g.opt.device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (n_tokens <= budget)
+    return after_launch(ipv::launch_passthrough(kept_idx_out, sh.S, n_tokens, budget, st),
+                        "pass-through kernel");
+  if (n_tokens > IPV_MAX_TOKENS)
+    return fail(IPV_EINVAL, "n_tokens %lld exceeds IPV_MAX_TOKENS", static_cast<long long>(n_tokens));
+  if (sh.rp >= budget)
+    return fail(IPV_EINVAL, "recent tokens r*p = %lld must be below budget %lld", static_cast<long long>(sh.rp),
+                static_cast<long long>(budget));
+
+  ipv::ScoreArgs a{};
+  a.k = k->buf[k->cur];
+  a.v = v->buf[v->cur];
+  a.patch_id = k->patch_id[k->cur];
+  a.n_slabs = sh.S;
+  a.cap = g.opt.token_capacity;
+  a.n_tokens = sh.N;
+  a.D = sh.D;
+  a.p = sh.p;
+  a.r = sh.r;
+  a.is_bf16 = g.opt.dtype == IPV_BF16;
+  a.m = g.m;
+  a.tar = g.tar;
+  a.van = g.van;
+  a.zero_recent = 0;
+  a.num_sms = g.num_sms;
+  prof_begin(0, st);
+  cudaError_t e = ipv::launch_recent_mean(a, st);
+  prof_end(0, st);
+  if (e != cudaSuccess) return cuda_fail(e, "recent-frame mean kernel");
+  prof_begin(1, st);
+  e = ipv::launch_score(a, st);
+  prof_end(1, st);
+  if (e != cudaSuccess) return cuda_fail(e, "scoring kernel");
+
+  ipv::SelectArgs sa{};
+  sa.tar = g.tar;
+  sa.van = g.van;
+  sa.n_slabs = sh.S;
+  sa.n_tokens = sh.N;
+  sa.rp = sh.rp;
+  sa.budget = budget;
+  split_budget(budget, tar_ratio, sh.rp, &sa.n_tar, &sa.n_van);
+  sa.kept = kept_idx_out;
+  prof_begin(2, st);
+  e = ipv::launch_select(sa, st);
+  prof_end(2, st);
+  if (e != cudaSuccess) return cuda_fail(e, "selection kernel");
+
+  ipv::GatherArgs ga{};
+  ga.k_src = k->buf[k->cur];
+  ga.v_src = v->buf[v->cur];
+  ga.k_dst = k->buf[1 - k->cur];
+  ga.v_dst = v->buf[1 - v->cur];
+  ga.pid_src = k->patch_id[k->cur];
+  ga.pid_dst = k->patch_id[1 - k->cur];
+  ga.kept = kept_idx_out;
+  ga.n_slabs = sh.S;
+  ga.cap = g.opt.token_capacity;
+  ga.budget = budget;
+  ga.row_bytes = sh.D * elem_bytes();
+  ga.p = sh.p;
+  ga.num_sms = g.num_sms;
+  prof_begin(3, st);
+  e = ipv::launch_gather(ga, st);
+  prof_end(3, st);
+  if (e != cudaSuccess) return cuda_fail(e, "compaction kernel");
+  k->cur = 1 - k->cur;
+  v->cur = 1 - v->cur;
+  return IPV_OK;
+}
+
+ipv_status ipv_profile_enable(int on) {
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  cudaSetDevice(g.opt.device);
+  // Create the events up front so that timed loops do not pay for it.
+  while (on && g.pool.size() < 4096) {
+    EventPair p;
+    if (cudaEventCreate(&p.start) != cudaSuccess || cudaEventCreate(&p.stop) != cudaSuccess)
+      return cuda_fail(cudaGetLastError(), "cudaEventCreate");
+    g.pool.push_back(p);
+  }
+  g.profiling = on != 0;
+  return IPV_OK;
+}
+
+ipv_status ipv_profile_collect(double ms_out[IPV_NUM_KERNELS], int64_t launches_out[IPV_NUM_KERNELS],
+                               int timeout_ms) {
+  if (!ms_out || !launches_out) return fail(IPV_EINVAL, "outputs must not be NULL");
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  cudaSetDevice(g.opt.device);
+  for (int id = 0; id < IPV_NUM_KERNELS; ++id) {
+    ms_out[id] = 0.0;
+    launches_out[id] = 0;
+  }
+  // Bounded wait for the last recorded stop event of every kernel id.
+  const int step_us = 200;
+  int waited_us = 0;
+  for (int id = 0; id < IPV_NUM_KERNELS; ++id) {
+    if (g.pending[id].empty()) continue;
+    for (;;) {
+      cudaError_t q = cudaEventQuery(g.pending[id].back().stop);
+      if (q == cudaSuccess) break;
+      if (q != cudaErrorNotReady) return cuda_fail(q, "cudaEventQuery");
+      if (waited_us >= timeout_ms * 1000) return fail(IPV_ETIMEOUT, "profiling events not complete after %d ms", timeout_ms);
+      struct timespec ts = {0, step_us * 1000};
+      nanosleep(&ts, nullptr);
+      waited_us += step_us;
+    }
+  }
+  for (int id = 0; id < IPV_NUM_KERNELS; ++id) {
+    for (auto& p : g.pending[id]) {
+      float ms = 0.0f;
+      cudaError_t e = cudaEventElapsedTime(&ms, p.start, p.stop);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+      ms_out[id] += ms;
+      launches_out[id] += 1;
+      g.pool.push_back(p);
+    }
+    g.pending[id].clear();
+  }
+  return IPV_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,128 @@
+// Internal declarations shared by the kernel translation units of libipv.so.
+// Not installed; the public interface is include/ipv.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ipv {
+
+constexpr int kHalfWarp = 16;        // lanes that cooperate on one 16-byte-chunked row
+constexpr float kNormEps = 1e-12f;   // cos(a,b) = a.b / (max|a|,eps)(max|b|,eps)
+constexpr int kSelectThreads = 1024;
+constexpr int kSelectBins = 2048;
+
+// ---------------------------------------------------------------- device helpers
+// 16-byte global load that bypasses L1 (each cache row is read once per kernel).
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+// 16-byte global store marked evict-first in L2.
+__device__ __forceinline__ void st_stream(void* p, uint4 v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+
+// Elements held by one 16-byte chunk, widened to fp32.
+template <typename T>
+struct Chunk;
+
+template <>
+struct Chunk<uint16_t> {  // bf16 bit patterns
+  static constexpr int kElems = 8;
+  __device__ __forceinline__ static void widen(uint4 c, float* x) {
+    const uint32_t w[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      x[2 * i] = __uint_as_float(w[i] << 16);
+      x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+  }
+};
+
+template <>
+struct Chunk<float> {
+  static constexpr int kElems = 4;
+  __device__ __forceinline__ static void widen(uint4 c, float* x) {
+    x[0] = __uint_as_float(c.x);
+    x[1] = __uint_as_float(c.y);
+    x[2] = __uint_as_float(c.z);
+    x[3] = __uint_as_float(c.w);
+  }
+};
+
+// Sum over the 16 lanes of a half-warp (every lane gets the total).
+__device__ __forceinline__ float halfwarp_sum(float x) {
+  x += __shfl_xor_sync(0xffffffffu, x, 8);
+  x += __shfl_xor_sync(0xffffffffu, x, 4);
+  x += __shfl_xor_sync(0xffffffffu, x, 2);
+  x += __shfl_xor_sync(0xffffffffu, x, 1);
+  return x;
+}
+
+// Order-preserving 32-bit key of a score: larger float -> larger key; -0 and
+// +0 are the same key; every NaN maps to 1, below every number (the smallest
+// number, -inf, maps to 0x007FFFFF). Keys 0 and 0xFFFFFFFF are never produced
+// and serve as "excluded" / "taken" marks in the selection kernel.
+__device__ __forceinline__ uint32_t score_key(float x) {
+  if (x != x) return 1u;
+  const uint32_t b = __float_as_uint(x + 0.0f);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// ---------------------------------------------------------------- host launchers
+struct ScoreArgs {
+  const void* k;            // [S][cap][D]
+  const void* v;
+  const uint16_t* patch_id; // [S][cap] or nullptr
+  int64_t n_slabs, cap, n_tokens;
+  int D, p, r;
+  int is_bf16;
+  float* m;                 // scratch [S][p][D] fp32
+  float* tar;               // [S][n_tokens]
+  float* van;
+  int zero_recent;          // write 0 to the recent-frame entries of tar/van
+  int num_sms;
+};
+
+cudaError_t launch_recent_mean(const ScoreArgs& a, cudaStream_t st);
+cudaError_t launch_score(const ScoreArgs& a, cudaStream_t st);
+size_t score_smem_bytes(int p, int D);
+cudaError_t score_prepare(int max_p, int max_D);
+
+struct SelectArgs {
+  const float* tar;   // [S][n_tokens]
+  const float* van;
+  int64_t n_slabs, n_tokens;
+  int64_t rp, n_tar, n_van, budget;
+  int32_t* kept;      // [S][budget]
+};
+
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
+cudaError_t launch_passthrough(int32_t* kept, int64_t n_slabs, int64_t n_tokens, int64_t budget,
+                               cudaStream_t st);
+size_t select_smem_bytes(int64_t n_tokens);
+cudaError_t select_prepare(int64_t max_tokens);
+
+struct GatherArgs {
+  const void* k_src;
+  const void* v_src;
+  void* k_dst;
+  void* v_dst;
+  const uint16_t* pid_src;  // nullptr: patch = n mod p
+  uint16_t* pid_dst;        // nullptr: not written
+  const int32_t* kept;      // [S][budget]
+  int64_t n_slabs, cap, budget;
+  int row_bytes, p;
+  int num_sms;
+};
+
+cudaError_t launch_gather(const GatherArgs& a, cudaStream_t st);
+
+}  // namespace ipv

@@ -1,0 +1,318 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Inputs are seeded synthetic caches (synth/); both sides read the same bytes.
+Scores, indices and compacted bytes are checked with the rules in parity.py.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from parity import assert_gather_exact, assert_scores_close, assert_selection_matches
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from paper_2506_15745_gb300 import ipv  # noqa: E402
+from paper_2506_15745_gb300.cache import PingPongCache  # noqa: E402
+
+
+def to_np(t):
+    t = t.contiguous()
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).cpu().numpy().view(np.uint16)
+    if t.dtype == torch.int16:
+        return t.cpu().numpy().view(np.uint16)
+    return t.cpu().numpy()
+
+
+def to_dev(a, dtype):
+    if dtype == "bf16":
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+@pytest.fixture(autouse=True)
+def _shutdown_after():
+    yield
+    torch.cuda.synchronize()
+    ipv.shutdown()
+
+
+def init_for(S, cap, D, p, dtype, recent_frames=0):
+    ipv.init(device=0, dtype=dtype, recent_frames=recent_frames, max_head_dim=D,
+             max_frame_tokens=p, max_slabs=S, token_capacity=cap)
+
+
+def check_pass(cache, L, H, N, gh, gw, budget, alpha, pid_valid, slabs=None):
+    """One compress pass on `cache` (live rows 0..N-1) checked end to end.
+    slabs: optional subset of slab indices for the oracle (large cases)."""
+    p = gh * gw
+    S, D = cache.n_slabs, cache.head_dim
+    r = ipv.recent_frames(N // p)
+    sel = np.arange(S) if slabs is None else np.asarray(slabs)
+    sel_t = torch.as_tensor(sel, device="cuda")
+    cache.n_tokens = N
+    k_src = to_np(cache.k_live.index_select(0, sel_t))
+    v_src = to_np(cache.v_live.index_select(0, sel_t))
+    pid_src = (to_np(cache.pid_live.index_select(0, sel_t))
+               if (pid_valid and cache.pid is not None) else None)
+    k_struct, v_struct = cache.structs(pid_valid)
+    tar_g = torch.empty((S, N), dtype=torch.float32, device="cuda")
+    van_g = torch.empty_like(tar_g)
+    has_past = r * p < N
+    if has_past:
+        ipv.score(k_struct, v_struct, L, H, D, N, gh, gw, tar_g, van_g)
+    kept_sel = torch.empty((S, budget), dtype=torch.int32, device="cuda")
+    if has_past:
+        ipv.select(tar_g, van_g, S, N, gh, gw, budget, alpha, kept_sel)
+    kept = torch.full((S, budget), -7, dtype=torch.int32, device="cuda")
+    cur_before = cache.cur
+    cache.compress(L, H, gh, gw, budget, alpha, kept, pid_valid=pid_valid)
+    torch.cuda.synchronize()
+    kept_np = to_np(kept.index_select(0, sel_t))
+    if N <= budget:  # pass-through
+        assert cache.cur == cur_before
+        want = np.array(list(range(N)) + [-1] * (budget - N), np.int32)
+        assert np.all(kept_np == want)
+        return None
+    assert cache.cur != cur_before
+    assert np.array_equal(to_np(kept_sel.index_select(0, sel_t)), kept_np)  # ipv_select == the pass
+    o_tar, o_van = oracle.scores(k_src, v_src, N, p, r, pid_src)
+    tg, vg = to_np(tar_g.index_select(0, sel_t)), to_np(van_g.index_select(0, sel_t))
+    errs = assert_scores_close(tg, vg, o_tar, o_van, N - r * p)
+    assert np.all(tg[:, N - r * p:] == 0) and np.all(vg[:, N - r * p:] == 0)
+    n_diff = assert_selection_matches(kept_np, tg, vg, o_tar, o_van, N, p, r, budget, alpha)
+    assert_gather_exact(k_src, to_np(cache.k_live.index_select(0, sel_t)), kept_np, budget)
+    assert_gather_exact(v_src, to_np(cache.v_live.index_select(0, sel_t)), kept_np, budget)
+    if cache.pid is not None:
+        pd = to_np(cache.pid_live.index_select(0, sel_t))[:, :budget]
+        want = (np.take_along_axis(pid_src, kept_np, 1) if pid_src is not None
+                else (kept_np % p).astype(np.uint16))
+        assert np.array_equal(pd, want)
+    return errs, n_diff
+
+
+def host_case(S, f, gh, gw, D, dtype, seed, static_frac=0.7, cap_extra=0):
+    w = synth.Workload("case", 1, S, D, dtype, gh, gw, f, 1, 0.5, static_frac=static_frac, seed=seed)
+    K, V = synth.host_generate(w)
+    cap = f * gh * gw + cap_extra
+    cache = PingPongCache(S, cap, D, dtype, patch_ids=True)
+    cache.k.zero_()
+    cache.v.zero_()
+    cache.k[0, :, :f * gh * gw] = to_dev(K, dtype)
+    cache.v[0, :, :f * gh * gw] = to_dev(V, dtype)
+    return cache
+
+
+def test_tiny_config():
+    """1 layer x 2 heads, D=64 fp32, 8 frames of 4x4, budget 48, alpha 0.5, seed 0."""
+    w = synth.CONFIGS["tiny"]
+    init_for(w.n_slabs, w.n_tokens, w.head_dim, w.p, w.dtype)
+    K, V = synth.host_generate(w)
+    cache = PingPongCache(w.n_slabs, w.n_tokens, w.head_dim, w.dtype)
+    cache.k[0] = to_dev(K, w.dtype)
+    cache.v[0] = to_dev(V, w.dtype)
+    errs, n_diff = check_pass(cache, w.n_layers, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w,
+                              w.budget, w.tar_ratio, pid_valid=False)
+    assert n_diff == 0
+    # The compacted half (with its patch ids) is a valid input for the next pass.
+    cache2 = PingPongCache(w.n_slabs, w.n_tokens, w.head_dim, w.dtype)
+    cache2.k[0] = to_dev(K, w.dtype)
+    cache2.v[0] = to_dev(V, w.dtype)
+    cache2.pid[0] = torch.arange(w.n_tokens, device="cuda").remainder(w.p).to(torch.int16)
+    check_pass(cache2, w.n_layers, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w, w.budget,
+               w.tar_ratio, pid_valid=True)
+    B = w.budget
+    assert torch.equal(cache2.k[1, :, :B], cache.k[1, :, :B])
+    assert torch.equal(cache2.pid[1, :, :B], cache.pid[1, :, :B])
+
+
+EDGE_CASES = [
+    # S, f, gh, gw, D, dtype, budget_fn(N, p, rp), alpha
+    (3, 12, 14, 14, 128, "bf16", lambda N, p, rp: N // 2 + 37, 0.5),      # ragged budget, many tiles
+    (5, 40, 1, 7, 64, "bf16", lambda N, p, rp: 150, 0.3),                 # half-warp lanes idle
+    (2, 16, 4, 4, 96, "bf16", lambda N, p, rp: rp + 1, 0.5),              # minimal budget
+    (3, 20, 2, 5, 128, "f32", lambda N, p, rp: N - 1, 0.7),               # evict one token
+    (4, 30, 1, 3, 32, "f32", lambda N, p, rp: 40, 0.0),                   # VaN only
+    (2, 16, 7, 7, 256, "bf16", lambda N, p, rp: 400, 1.0),                # TaR only, 2 chunks/lane
+    (2, 10, 3, 3, 512, "bf16", lambda N, p, rp: 50, 0.5),                 # 4 chunks/lane
+    (2, 10, 3, 3, 512, "f32", lambda N, p, rp: 50, 0.5),                  # 8 chunks/lane
+    (1, 9, 1, 1, 64, "bf16", lambda N, p, rp: 4, 0.5),                    # p = 1
+    (2, 8, 4, 4, 64, "f32", lambda N, p, rp: N, 0.5),                     # pass-through N == C
+    (2, 8, 4, 4, 64, "f32", lambda N, p, rp: N + 9, 0.5),                 # pass-through N < C
+]
+
+
+@pytest.mark.parametrize("case", range(len(EDGE_CASES)))
+def test_edge_shapes(case):
+    S, f, gh, gw, D, dtype, budget_fn, alpha = EDGE_CASES[case]
+    p = gh * gw
+    N = f * p
+    cap = N + 64
+    budget = budget_fn(N, p, oracle.recent_frames(f) * p)
+    assert budget <= cap
+    init_for(S, cap, D, p, dtype)
+    cache = host_case(S, f, gh, gw, D, dtype, seed=100 + case, cap_extra=64)
+    check_pass(cache, 1, S, N, gh, gw, budget, alpha, pid_valid=False)
+
+
+@pytest.mark.parametrize("r", [1, 3])
+def test_recent_frames_override(r):
+    S, f, gh, gw, D = 3, 10, 4, 5, 128
+    init_for(S, f * gh * gw, D, gh * gw, "bf16", recent_frames=r)
+    assert ipv.recent_frames(f) == r
+    cache = host_case(S, f, gh, gw, D, "bf16", seed=7)
+    check_pass(cache, 1, S, f * gh * gw, gh, gw, 90, 0.5, pid_valid=False)
+
+
+def test_patch_ids_are_followed():
+    """Past rows shuffled together with their patch ids score as before."""
+    S, f, gh, gw, D = 2, 12, 3, 4, 128
+    p, N = gh * gw, f * gh * gw
+    init_for(S, N, D, p, "bf16")
+    cache = host_case(S, f, gh, gw, D, "bf16", seed=11)
+    r = ipv.recent_frames(f)
+    n_past = N - r * p
+    perm = torch.from_numpy(np.random.default_rng(3).permutation(n_past)).cuda()
+    cache.k[0, :, :n_past] = cache.k[0, :, perm].clone()
+    cache.v[0, :, :n_past] = cache.v[0, :, perm].clone()
+    pid = torch.arange(N, device="cuda").remainder(p)
+    pid[:n_past] = perm.remainder(p)
+    cache.pid[0] = pid.to(torch.int16).expand(S, N)
+    check_pass(cache, 1, S, N, gh, gw, N // 2, 0.5, pid_valid=True)
+
+
+def test_select_exact_on_ties_nan_and_signed_zero():
+    """Step (iii) alone on crafted fp32 scores: bit-exact against the oracle."""
+    rng = np.random.default_rng(5)
+    S, f, p = 6, 20, 7
+    N = f * p
+    init_for(S, N, 64, p, "f32")
+    tar = (rng.integers(-3, 3, size=(S, N)) / 2).astype(np.float32)   # heavy ties
+    van = rng.integers(0, 4, size=(S, N)).astype(np.float32)
+    tar[0, :50] = -1.0                    # all equal
+    tar[1, ::3] = np.nan                  # NaN ranks lowest
+    van[2, ::4] = np.nan
+    tar[3, ::2] = -0.0                    # -0 and +0 tie, broken by index
+    tar[3, 1::2] = 0.0
+    van[4] = 2.5                          # all VaN equal
+    for budget, alpha in [(60, 0.5), (30, 0.9), (139, 0.5), (25, 0.0), (70, 1.0)]:
+        r = oracle.recent_frames(f)
+        kept = torch.empty((S, budget), dtype=torch.int32, device="cuda")
+        ipv.select(torch.from_numpy(tar).cuda(), torch.from_numpy(van).cuda(), S, N, 1, p,
+                   budget, alpha, kept)
+        want = oracle.select(tar.astype(np.float64), van.astype(np.float64), N, p, r, budget,
+                             float(np.float32(alpha)))
+        assert np.array_equal(to_np(kept), want), (budget, alpha)
+
+
+def test_invalid_arguments_are_rejected():
+    S, f, gh, gw, D = 2, 8, 4, 4, 64
+    p, N = gh * gw, f * gh * gw
+    init_for(S, N, D, p, "f32")
+    cache = host_case(S, f, gh, gw, D, "f32", seed=1)
+    kept = torch.empty((S, N), dtype=torch.int32, device="cuda")
+    k, v = cache.structs(False)
+    bad = [
+        dict(n_tokens=N + p),                 # above token_capacity
+        dict(n_tokens=N - 1),                 # not whole frames
+        dict(budget=p),                       # r p >= budget
+        dict(tar_ratio=1.5),
+        dict(tar_ratio=float("nan")),
+        dict(head_dim=D * 2),                 # above max_head_dim
+        dict(n_layers=2),                     # above max_slabs
+        dict(frame_grid_w=gw * 2, n_tokens=N),  # above max_frame_tokens
+    ]
+    for over in bad:
+        args = dict(n_layers=1, n_kv_heads=S, head_dim=D, n_tokens=N, frame_grid_h=gh,
+                    frame_grid_w=gw, budget=N // 2, tar_ratio=0.5)
+        args.update(over)
+        with pytest.raises(ipv.IpvError) as ei:
+            ipv.compress(k, v, args["n_layers"], args["n_kv_heads"], args["head_dim"],
+                         args["n_tokens"], args["frame_grid_h"], args["frame_grid_w"],
+                         args["budget"], args["tar_ratio"], kept)
+        assert ei.value.status == ipv.IPV_EINVAL, over
+        assert k.cur == 0 and v.cur == 0
+
+
+def _device_config(name, patch_ids=False):
+    w = synth.CONFIGS[name]
+    init_for(w.slabs_per_stream, w.n_tokens, w.head_dim, w.p, w.dtype)
+    cache = PingPongCache(w.slabs_per_stream, w.n_tokens, w.head_dim, w.dtype, patch_ids=patch_ids)
+    synth.device_generate(w, cache.k[0], cache.v[0])
+    return w, cache
+
+
+@pytest.mark.parametrize("name", ["llava", "qwen"])
+def test_full_config(name):
+    """Configs at full size (28 layers x 4 KV heads), every slab checked."""
+    w, cache = _device_config(name, patch_ids=True)
+    check_pass(cache, w.n_layers, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w, w.budget,
+               w.tar_ratio, pid_valid=False)
+
+
+def test_streaming_run():
+    """1 h at 1 fps at the LLaVA shape: 16 frames appended per step, a pass
+    whenever the cache holds 9408 tokens. Every pass keeps the invariants; the
+    first, a middle and the last pass are checked against the oracle on 16
+    sampled slabs (past rows then carry patch ids from earlier passes)."""
+    w = synth.CONFIGS["stream"]
+    S, p = w.slabs_per_stream, w.p
+    init_for(S, w.n_tokens, w.head_dim, p, w.dtype)
+    cache = PingPongCache(S, w.n_tokens, w.head_dim, w.dtype, patch_ids=True)
+    gen = synth.DeviceGenerator(w, S)
+    kept = torch.empty((S, w.budget), dtype=torch.int32, device="cuda")
+    n_passes = (w.stream_frames - w.n_frames) // w.append_frames + 1
+    check_at = {0, n_passes // 2, n_passes - 1}
+    sample = np.random.default_rng(0).choice(S, 16, replace=False)
+    r = ipv.recent_frames(w.n_frames)
+    passes = frames = 0
+    first = True
+    while frames < w.stream_frames:
+        nf = min(w.append_frames, w.stream_frames - frames)
+        row0 = cache.n_tokens
+        gen.fill(cache.k_live, cache.v_live, row0, nf)
+        cache.pid_live[:, row0:row0 + nf * p] = (
+            torch.arange(nf * p, device="cuda").remainder(p).to(torch.int16))
+        cache.n_tokens += nf * p
+        frames += nf
+        if cache.n_tokens >= w.n_tokens:
+            assert cache.n_tokens == w.n_tokens
+            if passes in check_at:
+                check_pass(cache, w.n_layers, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w,
+                           w.budget, w.tar_ratio, pid_valid=True, slabs=sample)
+            else:
+                cache.compress(w.n_layers, w.n_kv_heads, w.grid_h, w.grid_w, w.budget,
+                               w.tar_ratio, kept, pid_valid=True)
+                kn = kept
+                assert torch.all(kn[:, 1:] > kn[:, :-1])
+                assert torch.equal(kn[:, -r * p:], torch.arange(w.n_tokens - r * p, w.n_tokens,
+                                                                device="cuda", dtype=torch.int32).expand(S, -1))
+            passes += 1
+            first = False
+    assert passes == n_passes == 223 and not first
+
+
+def test_large_config_sampled():
+    """8 streams x 80 layers x 8 KV heads, 32768 -> 24576 tokens (~86 GB of
+    K/V plus the second ping-pong half). 8 sampled slabs checked."""
+    w = synth.CONFIGS["large"]
+    S = w.n_slabs
+    need = 2 * 2 * S * w.n_tokens * w.head_dim * 2 + 3 * S * w.n_tokens * 4 + (8 << 30)
+    free, _ = torch.cuda.mem_get_info()
+    if free < need:
+        pytest.skip(f"needs {need / 2**30:.0f} GiB free, {free / 2**30:.0f} GiB available")
+    init_for(S, w.n_tokens, w.head_dim, w.p, w.dtype)
+    cache = PingPongCache(S, w.n_tokens, w.head_dim, w.dtype, patch_ids=False)
+    per = w.slabs_per_stream
+    for st in range(w.n_streams):
+        synth.device_generate(w, cache.k[0, st * per:(st + 1) * per],
+                              cache.v[0, st * per:(st + 1) * per], stream=st)
+    sample = np.random.default_rng(1).choice(S, 8, replace=False)
+    try:
+        check_pass(cache, w.n_streams * w.n_layers, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w,
+                   w.budget, w.tar_ratio, pid_valid=False, slabs=sample)
+    finally:
+        del cache
+        torch.cuda.empty_cache()

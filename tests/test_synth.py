@@ -1,0 +1,50 @@
+"""The seeded input generator follows its stated recipe (CPU)."""
+import numpy as np
+
+import synth
+
+
+def test_philox_known_answers():
+    """Philox4x32-10 known-answer vectors published with Random123."""
+    r = synth.philox4x32_10((0, 0, 0, 0), (0, 0))
+    assert [int(x) for x in r] == [0x6627E8D5, 0xE169C58D, 0xBC57AC4C, 0x9B00DBD8]
+    r = synth.philox4x32_10((0xFFFFFFFF,) * 4, (0xFFFFFFFF,) * 2)
+    assert [int(x) for x in r] == [0x408F276D, 0x41C83B0E, 0xA20BC7C6, 0x6D5451FD]
+    r = synth.philox4x32_10((0x243F6A88, 0x85A308D3, 0x13198A2E, 0x03707344),
+                            (0xA4093822, 0x299F31D0))
+    assert [int(x) for x in r] == [0xD16CFE09, 0x94FDCCEB, 0x5001E420, 0x24126EA1]
+
+
+def test_patch_kinds():
+    for name in ("tiny", "llava", "qwen"):
+        w = synth.CONFIGS[name]
+        rho = synth.patch_rho(w)
+        assert (rho == np.float32(w.rho_static)).sum() == int(np.floor(w.static_frac * w.p))
+        assert np.array_equal(rho, synth.patch_rho(w))          # seeded
+    w = synth.CONFIGS["llava"]
+    assert not np.array_equal(synth.patch_rho(w, 0), synth.patch_rho(w, 1))
+
+
+def test_key_and_value_statistics():
+    w = synth.CONFIGS["llava"].scaled(n_layers=1, n_kv_heads=2, n_frames=24, head_dim=64)
+    K, V = synth.host_generate(w)
+    K = synth.bf16_bits_to_f32(K).astype(np.float64).reshape(2, w.n_frames, w.p, w.head_dim)
+    V = synth.bf16_bits_to_f32(V).astype(np.float64)
+    rho = synth.patch_rho(w)
+    for kind in (w.rho_static, w.rho_dynamic):
+        q = np.nonzero(rho == np.float32(kind))[0]
+        a, b = K[:, :-1, q].ravel(), K[:, 1:, q].ravel()
+        assert abs(np.corrcoef(a, b)[0, 1] - kind) < 0.05
+    dyn = np.nonzero(rho == np.float32(w.rho_dynamic))[0]
+    var = K[:, :, dyn].var()
+    assert abs(var - 1 / (1 - w.rho_dynamic ** 2)) < 0.1          # stationary variance
+    lognorm = np.log(np.linalg.norm(V, axis=-1)).ravel()
+    assert abs(lognorm.mean()) < 0.03 and abs(lognorm.std() - w.value_sigma) < 0.03
+
+
+def test_bf16_rounding_is_nearest_even():
+    x = np.array([1.0, 1.00390625, 1.01171875, -2.5, 3.0e-3], np.float32)
+    b = synth.to_bf16_bits(x)
+    back = synth.bf16_bits_to_f32(b)
+    assert b[1] == 0x3F80 and b[2] == 0x3F82       # ties to even
+    assert np.all(np.abs(back - x) <= np.abs(x) * 2 ** -8)
