@@ -7,16 +7,16 @@
 
 namespace ipv {
 
-constexpr int kHalfWarp = 16;        // lanes that cooperate on one 16-byte-chunked row
 constexpr float kNormEps = 1e-12f;   // cos(a,b) = a.b / (max|a|,eps)(max|b|,eps)
 constexpr int kSelectThreads = 1024;
 constexpr int kSelectBins = 2048;
 
 // ---------------------------------------------------------------- device helpers
-// 16-byte global load that bypasses L1 (each cache row is read once per kernel).
+// 16-byte global load that bypasses L1 (each cache row is read once per
+// kernel). Only for data no thread writes while the kernel runs.
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
   uint4 r;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
                : "l"(p));
   return r;
@@ -33,38 +33,31 @@ __device__ __forceinline__ void st_stream(void* p, uint4 v) {
 template <typename T>
 struct Chunk;
 
+// Elements are handled in consecutive pairs so that sums can use the packed
+// fp32 FMA (each lane of fma.rn.f32x2 is an ordinary IEEE fma).
 template <>
 struct Chunk<uint16_t> {  // bf16 bit patterns
   static constexpr int kElems = 8;
-  __device__ __forceinline__ static void widen(uint4 c, float* x) {
+  static constexpr int kPairs = 4;
+  __device__ __forceinline__ static void widen2(uint4 c, float2* x) {
     const uint32_t w[4] = {c.x, c.y, c.z, c.w};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      x[2 * i] = __uint_as_float(w[i] << 16);
-      x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-    }
+    for (int i = 0; i < 4; ++i)
+      x[i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
   }
 };
 
 template <>
 struct Chunk<float> {
   static constexpr int kElems = 4;
-  __device__ __forceinline__ static void widen(uint4 c, float* x) {
-    x[0] = __uint_as_float(c.x);
-    x[1] = __uint_as_float(c.y);
-    x[2] = __uint_as_float(c.z);
-    x[3] = __uint_as_float(c.w);
+  static constexpr int kPairs = 2;
+  __device__ __forceinline__ static void widen2(uint4 c, float2* x) {
+    x[0] = make_float2(__uint_as_float(c.x), __uint_as_float(c.y));
+    x[1] = make_float2(__uint_as_float(c.z), __uint_as_float(c.w));
   }
 };
 
-// Sum over the 16 lanes of a half-warp (every lane gets the total).
-__device__ __forceinline__ float halfwarp_sum(float x) {
-  x += __shfl_xor_sync(0xffffffffu, x, 8);
-  x += __shfl_xor_sync(0xffffffffu, x, 4);
-  x += __shfl_xor_sync(0xffffffffu, x, 2);
-  x += __shfl_xor_sync(0xffffffffu, x, 1);
-  return x;
-}
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 
 // Order-preserving 32-bit key of a score: larger float -> larger key; -0 and
 // +0 are the same key; every NaN maps to 1, below every number (the smallest

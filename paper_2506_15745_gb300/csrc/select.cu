@@ -4,16 +4,18 @@
 // the r*p recent tokens are kept; the n_tar past tokens of highest s_TaR are
 // taken; then the n_van past tokens of highest s_VaN among those TaR left
 // (Algorithm 2 forces TaR picks to max(VaN) before its final TopK, which is
-// the same as excluding them). Ties go to the lower token index. The kept
-// set is written as ascending row indices.
+// the same as excluding them). Ties go to the lower token index; NaN ranks
+// below every number. The kept set is written as ascending row indices.
 //
-// One 1024-thread CTA per slab; the scores are turned into order-preserving
-// uint32 keys held in shared memory. A top-k threshold is found by repeated
-// histogramming: the current key window [lo, hi] is split into 2048 equal
-// integer bins, the bin holding the k-th largest key becomes the next window
-// (at most 3 rounds for 32-bit keys). Tokens above the threshold key are
-// taken, and of the tokens equal to it the lowest-index ones, counted with a
-// block-wide prefix sum in index order.
+// One 1024-thread CTA per slab; scores live in shared memory as
+// order-preserving uint32 keys. Each stage finds its k winners without a
+// sort: a 2048-bin histogram that is linear in the score value over
+// [min, max] of the candidates (a monotone map, so every bin above the one
+// holding the k-th winner is taken whole); the candidates of that boundary
+// bin, usually a few dozen, are ranked exactly against each other with the
+// index tie-break. A boundary bin of more than 1024 candidates (heavy ties
+// or extreme clustering) falls back to an exact search over integer key
+// windows with ties counted by a block-wide prefix sum in index order.
 #include "ipv_common.cuh"
 
 namespace ipv {
@@ -21,13 +23,33 @@ namespace {
 
 constexpr uint32_t kTaken = 0xFFFFFFFFu;    // VaN pick (never a score key)
 constexpr uint32_t kExcluded = 0u;          // TaR pick, excluded from the VaN stage
+constexpr uint32_t kNanKey = 1u;            // score_key of every NaN
 constexpr uint32_t kNoBin = 0xFFFFFFFFu;
+constexpr int kListMax = kSelectThreads;    // boundary candidates ranked directly
 
 struct BlockShared {
   uint32_t warp_a[32];
   uint32_t warp_b[32];
+  float warp_f[32];
+  float warp_g[32];
   uint32_t bcast[8];
+  float fcast[2];
+  uint32_t list_n;
 };
+
+// Candidates of a stage: real score keys (NaN included), not yet taken.
+__device__ __forceinline__ bool is_cand(uint32_t k) { return k != kExcluded && k != kTaken; }
+
+// Inverse of score_key for keys >= 2.
+__device__ __forceinline__ float key_value(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+// Monotone non-decreasing bin of a score in [vmin, vmax].
+__device__ __forceinline__ int value_bin(float v, float vmin, float scale) {
+  const int b = static_cast<int>((v - vmin) * scale);
+  return b < kSelectBins - 1 ? b : kSelectBins - 1;
+}
 
 __device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v) {
   const int lane = threadIdx.x & 31;
@@ -58,7 +80,7 @@ __device__ uint32_t block_excl_scan(uint32_t v, uint32_t* total, BlockShared& sh
   return out;
 }
 
-// Block-wide min and max of candidate keys (key >= 1); broadcast to all.
+// Block-wide min/max of uint32 keys; broadcast to all threads.
 __device__ void block_minmax(uint32_t lo, uint32_t hi, uint32_t* out_lo, uint32_t* out_hi,
                              BlockShared& sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -91,32 +113,95 @@ __device__ void block_minmax(uint32_t lo, uint32_t hi, uint32_t* out_lo, uint32_
   __syncthreads();
 }
 
-// Threshold of the k largest candidate keys (candidates: key >= 1) among
-// key[0..n). The k winners are: every candidate with key > *T, plus the
-// *take_eq lowest-index candidates with key == *T. *cnt_eq is the number of
-// candidates with key == *T (only meaningful when *take_eq > 0).
-// Requires 1 <= k <= number of candidates (n_cand).
-__device__ void find_threshold(const uint32_t* key, int n, uint32_t k, uint32_t n_cand,
-                               uint32_t* hist, BlockShared& sh, uint32_t* T, uint32_t* take_eq,
-                               uint32_t* cnt_eq) {
-  if (k >= n_cand) {  // every candidate is taken
-    *T = 0u;
-    *take_eq = 0u;
-    *cnt_eq = 0u;
-    return;
+// Value range and NaN count of a stage's candidates.
+struct Stats {
+  float vmin, vmax;
+  uint32_t n_nan;
+};
+
+__device__ __forceinline__ void stats_add(Stats& st, float v) {
+  if (v != v) {
+    ++st.n_nan;
+  } else {
+    st.vmin = fminf(st.vmin, v);
+    st.vmax = fmaxf(st.vmax, v);
   }
-  uint32_t lo = 0xFFFFFFFFu, hi = 0u;
-  for (int i = threadIdx.x; i < n; i += kSelectThreads) {
-    const uint32_t x = key[i];
-    if (x >= 1u) {
-      lo = min(lo, x);
-      hi = max(hi, x);
+}
+
+__device__ Stats block_stats(Stats st, BlockShared& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    st.vmin = fminf(st.vmin, __shfl_xor_sync(0xffffffffu, st.vmin, off));
+    st.vmax = fmaxf(st.vmax, __shfl_xor_sync(0xffffffffu, st.vmax, off));
+    st.n_nan += __shfl_xor_sync(0xffffffffu, st.n_nan, off);
+  }
+  if (lane == 0) {
+    sh.warp_f[warp] = st.vmin;
+    sh.warp_g[warp] = st.vmax;
+    sh.warp_a[warp] = st.n_nan;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    st.vmin = sh.warp_f[lane];
+    st.vmax = sh.warp_g[lane];
+    st.n_nan = sh.warp_a[lane];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      st.vmin = fminf(st.vmin, __shfl_xor_sync(0xffffffffu, st.vmin, off));
+      st.vmax = fmaxf(st.vmax, __shfl_xor_sync(0xffffffffu, st.vmax, off));
+      st.n_nan += __shfl_xor_sync(0xffffffffu, st.n_nan, off);
+    }
+    if (lane == 0) {
+      sh.fcast[0] = st.vmin;
+      sh.fcast[1] = st.vmax;
+      sh.bcast[0] = st.n_nan;
     }
   }
-  block_minmax(lo, hi, &lo, &hi, sh);
-  uint32_t k_rem = k, cnt = n_cand;
-  // The window shrinks at least 2048-fold per round, so 32-bit keys converge
-  // in 4 rounds; the hard limit only guards against a broken invariant.
+  __syncthreads();
+  Stats out{sh.fcast[0], sh.fcast[1], sh.bcast[0]};
+  __syncthreads();
+  return out;
+}
+
+// Finds, from the histogram, the bin holding the k-th largest candidate
+// (bins scanned from the top). Thread t owns bins 2047-2t and 2046-2t.
+// Returns the bin (kNoBin if the histogram holds fewer than k), the count of
+// candidates in higher bins and the bin's own count.
+__device__ void boundary_bin(const uint32_t* hist, uint32_t k, BlockShared& sh, uint32_t* bsel,
+                             uint32_t* above, uint32_t* cnt_b) {
+  const int ba = kSelectBins - 1 - 2 * static_cast<int>(threadIdx.x), bb = ba - 1;
+  const uint32_t ha = hist[ba], hb = hist[bb];
+  if (threadIdx.x == 0) sh.bcast[2] = kNoBin;  // published by the scan's barriers
+  uint32_t tot;
+  const uint32_t above_a = block_excl_scan(ha + hb, &tot, sh);
+  const uint32_t above_b = above_a + ha;
+  if (above_a < k && k <= above_a + ha) {
+    sh.bcast[2] = ba;
+    sh.bcast[3] = above_a;
+    sh.bcast[4] = ha;
+  } else if (above_b < k && k <= above_b + hb) {
+    sh.bcast[2] = bb;
+    sh.bcast[3] = above_b;
+    sh.bcast[4] = hb;
+  }
+  __syncthreads();
+  *bsel = sh.bcast[2];
+  *above = sh.bcast[3];
+  *cnt_b = sh.bcast[4];
+  __syncthreads();
+}
+
+// Exact threshold search over integer key windows, starting from the window
+// [lo, hi] that holds cnt candidates of which the k largest are wanted (all
+// candidates above hi are taken already). On return the winners are the
+// candidates with key > *T plus the *take lowest-index ones with key == *T;
+// *cnt_eq counts the candidates equal to *T. The window shrinks at least
+// 2048-fold per round (4 rounds for 32-bit keys); the hard round limit only
+// guards against a broken invariant.
+__device__ void window_search(const uint32_t* key, int n, uint32_t lo, uint32_t hi, uint32_t k,
+                              uint32_t cnt, uint32_t* hist, BlockShared& sh, uint32_t* T,
+                              uint32_t* take_eq, uint32_t* cnt_eq) {
   for (int round = 0; round < 8; ++round) {
     if (lo == hi) break;
     const uint64_t W = static_cast<uint64_t>(hi - lo) + 1u;
@@ -128,33 +213,15 @@ __device__ void find_threshold(const uint32_t* key, int n, uint32_t k, uint32_t 
         atomicAdd(&hist[(static_cast<uint64_t>(x - lo) * kSelectBins) / W], 1u);
     }
     __syncthreads();
-    // Thread t owns bins 2047-2t and 2046-2t (descending); an exclusive scan
-    // gives the count of candidates in the bins above them.
-    const int ba = kSelectBins - 1 - 2 * threadIdx.x, bb = ba - 1;
-    const uint32_t ha = hist[ba], hb = hist[bb];
-    if (threadIdx.x == 0) sh.bcast[2] = kNoBin;  // published by the scan's barriers
-    uint32_t tot;
-    const uint32_t above_a = block_excl_scan(ha + hb, &tot, sh);
-    const uint32_t above_b = above_a + ha;
-    if (above_a < k_rem && k_rem <= above_a + ha) {
-      sh.bcast[2] = ba;
-      sh.bcast[3] = above_a;
-      sh.bcast[4] = ha;
-    } else if (above_b < k_rem && k_rem <= above_b + hb) {
-      sh.bcast[2] = bb;
-      sh.bcast[3] = above_b;
-      sh.bcast[4] = hb;
-    }
-    __syncthreads();
-    const uint32_t bsel = sh.bcast[2], above = sh.bcast[3], cnt_b = sh.bcast[4];
-    __syncthreads();
-    if (bsel == kNoBin) break;  // fewer candidates than k_rem: cannot happen
-    k_rem -= above;
+    uint32_t bsel, above, cnt_b;
+    boundary_bin(hist, k, sh, &bsel, &above, &cnt_b);
+    if (bsel == kNoBin) break;  // fewer candidates than k: cannot happen
+    k -= above;
     // Keys x with floor((x-lo)*2048/W) == bsel form [lo + ceil(bsel W/2048), lo + ceil((bsel+1) W/2048) - 1].
     const uint32_t lo_b = lo + static_cast<uint32_t>((bsel * W + kSelectBins - 1) / kSelectBins);
     const uint32_t hi_b =
         lo + static_cast<uint32_t>(((bsel + 1) * W + kSelectBins - 1) / kSelectBins) - 1u;
-    if (cnt_b == k_rem) {  // the whole bin is taken: threshold just below it
+    if (cnt_b == k) {  // the whole bin is taken: threshold just below it
       *T = lo_b - 1u;
       *take_eq = 0u;
       *cnt_eq = 0u;
@@ -165,13 +232,115 @@ __device__ void find_threshold(const uint32_t* key, int n, uint32_t k, uint32_t 
     cnt = cnt_b;
   }
   *T = lo;
-  *take_eq = k_rem;
+  *take_eq = k;
   *cnt_eq = cnt;
 }
 
+// How a stage's winners are recognised in the marking pass (block-uniform).
+struct Plan {
+  int mode;  // 0 none, 1 every candidate, 2 key threshold, 3 value bin (+ pre-marked)
+  uint32_t T, take, cnt_eq;
+  int bthr;
+  float vmin, scale;
+};
+
+// Decides a stage taking the k best of n_cand candidates. Boundary-bin
+// winners found by direct ranking are marked in place with `mark`.
+__device__ Plan plan_stage(uint32_t* key, int n, uint32_t k, uint32_t n_cand, Stats st,
+                           uint32_t mark, uint32_t* hist, uint32_t* list_key, uint32_t* list_idx,
+                           BlockShared& sh) {
+  Plan P{};
+  if (k == 0u) return P;
+  if (k >= n_cand) {
+    P.mode = 1;
+    return P;
+  }
+  const uint32_t n_num = n_cand - st.n_nan;
+  P.mode = 2;
+  if (k > n_num) {  // every number, then the lowest-index NaNs
+    P.T = kNanKey;
+    P.take = k - n_num;
+    P.cnt_eq = st.n_nan;
+    return P;
+  }
+  if (st.vmin == st.vmax) {  // all numbers equal
+    P.T = score_key(st.vmin);
+    P.take = k;
+    P.cnt_eq = n_num;
+    return P;
+  }
+  const float range = st.vmax - st.vmin;
+  const float scale = static_cast<float>(kSelectBins) / range;
+  uint32_t lo = score_key(st.vmin), hi = score_key(st.vmax), k_rem = k, cnt = n_num;
+  if (range < INFINITY && scale < INFINITY) {
+    for (int b = threadIdx.x; b < kSelectBins; b += kSelectThreads) hist[b] = 0u;
+    if (threadIdx.x == 0) sh.list_n = 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < n; i += kSelectThreads) {
+      const uint32_t x = key[i];
+      if (is_cand(x) && x != kNanKey) atomicAdd(&hist[value_bin(key_value(x), st.vmin, scale)], 1u);
+    }
+    __syncthreads();
+    uint32_t bsel, above, cnt_b;
+    boundary_bin(hist, k, sh, &bsel, &above, &cnt_b);
+    if (bsel != kNoBin) {
+      k_rem = k - above;
+      P.mode = 3;
+      P.vmin = st.vmin;
+      P.scale = scale;
+      if (cnt_b == k_rem) {  // the whole boundary bin is taken
+        P.bthr = static_cast<int>(bsel) - 1;
+        return P;
+      }
+      P.bthr = static_cast<int>(bsel);
+      if (cnt_b <= static_cast<uint32_t>(kListMax)) {
+        for (int i = threadIdx.x; i < n; i += kSelectThreads) {
+          const uint32_t x = key[i];
+          if (is_cand(x) && x != kNanKey &&
+              value_bin(key_value(x), st.vmin, scale) == static_cast<int>(bsel)) {
+            const uint32_t j = atomicAdd(&sh.list_n, 1u);
+            if (j < static_cast<uint32_t>(kListMax)) {
+              list_key[j] = x;
+              list_idx[j] = static_cast<uint32_t>(i);
+            }
+          }
+        }
+        __syncthreads();
+        const uint32_t m = min(sh.list_n, static_cast<uint32_t>(kListMax));
+        if (threadIdx.x < m) {
+          const uint32_t kt = list_key[threadIdx.x], it = list_idx[threadIdx.x];
+          uint32_t rank = 0u;
+          for (uint32_t j = 0; j < m; ++j) {
+            const uint32_t kj = list_key[j];
+            rank += (kj > kt || (kj == kt && list_idx[j] < it)) ? 1u : 0u;
+          }
+          if (rank < k_rem) key[it] = mark;
+        }
+        __syncthreads();
+        return P;
+      }
+      // Too many candidates in the bin: exact search inside its key range.
+      uint32_t blo = 0xFFFFFFFFu, bhi = 0u;
+      for (int i = threadIdx.x; i < n; i += kSelectThreads) {
+        const uint32_t x = key[i];
+        if (is_cand(x) && x != kNanKey &&
+            value_bin(key_value(x), st.vmin, scale) == static_cast<int>(bsel)) {
+          blo = min(blo, x);
+          bhi = max(bhi, x);
+        }
+      }
+      block_minmax(blo, bhi, &lo, &hi, sh);
+      cnt = cnt_b;
+    }
+  }
+  P.mode = 2;
+  window_search(key, n, lo, hi, k_rem, cnt, hist, sh, &P.T, &P.take, &P.cnt_eq);
+  return P;
+}
+
 // Rank-among-ties bookkeeping: each thread walks the contiguous chunk
-// [c0, c1) of indices; returns the number of candidates equal to T in the
-// chunks of lower-numbered threads.
+// [c0, c1) of indices; returns the number of keys equal to T in the chunks of
+// lower-numbered threads.
 __device__ uint32_t ties_before(const uint32_t* key, int c0, int c1, uint32_t T, BlockShared& sh) {
   uint32_t mine = 0u;
   for (int i = c0; i < c1; ++i) mine += (key[i] == T) ? 1u : 0u;
@@ -179,9 +348,43 @@ __device__ uint32_t ties_before(const uint32_t* key, int c0, int c1, uint32_t T,
   return block_excl_scan(mine, &tot, sh);
 }
 
+// Per-thread walker of a plan over the chunk [c0, c1) in index order.
+struct Picker {
+  Plan P;
+  uint32_t mark, rank;
+  bool all_ties;
+  __device__ bool pick(uint32_t x) {
+    if (x == mark) return true;  // ranked winner of the boundary bin
+    if (!is_cand(x)) return false;
+    switch (P.mode) {
+      case 1: return true;
+      case 2:
+        if (x > P.T) return true;
+        if (x == P.T) return all_ties || (rank++ < P.take);
+        return false;
+      case 3: return x != kNanKey && value_bin(key_value(x), P.vmin, P.scale) > P.bthr;
+      default: return false;
+    }
+  }
+};
+
+__device__ Picker make_picker(const uint32_t* key, int c0, int c1, const Plan& P, uint32_t mark,
+                              BlockShared& sh) {
+  Picker pk{P, mark, 0u, true};
+  if (P.mode == 2 && P.take > 0u && P.take < P.cnt_eq) {
+    pk.all_ties = false;
+    pk.rank = ties_before(key, c0, c1, P.T, sh);
+  } else if (P.mode == 2 && P.take == 0u) {
+    pk.all_ties = false;  // nothing equal to T is taken
+  }
+  return pk;
+}
+
 __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a) {
   extern __shared__ uint32_t sm_key[];
   __shared__ BlockShared sh;
+  __shared__ uint32_t list_key[kListMax];
+  __shared__ uint32_t list_idx[kListMax];
   const int n_past = static_cast<int>(a.n_tokens - a.rp);
   uint32_t* key = sm_key;
   uint32_t* hist = sm_key + ((n_past + 3) & ~3);
@@ -193,39 +396,43 @@ __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a)
   const int c1 = min(n_past, c0 + chunk);
 
   // TaR stage over all past tokens.
-  for (int i = threadIdx.x; i < n_past; i += kSelectThreads) key[i] = score_key(tar[i]);
-  __syncthreads();
-  uint32_t T = 0xFFFFFFFFu, take = 0u, cnt_eq = 0u;  // default: nothing taken
-  if (a.n_tar > 0)
-    find_threshold(key, n_past, static_cast<uint32_t>(a.n_tar), static_cast<uint32_t>(n_past),
-                   hist, sh, &T, &take, &cnt_eq);
-  uint32_t rank = (take > 0u && take < cnt_eq) ? ties_before(key, c0, c1, T, sh) : 0u;
-  const bool all_ties = take >= cnt_eq;
-  for (int i = c0; i < c1; ++i) {
-    const uint32_t x = key[i];
-    bool pick = x > T && a.n_tar > 0;
-    if (x == T && take > 0u) pick = all_ties || (rank++ < take);
-    key[i] = pick ? kExcluded : score_key(van[i]);
+  Stats st{INFINITY, -INFINITY, 0u};
+  for (int i = threadIdx.x; i < n_past; i += kSelectThreads) {
+    const float v = tar[i] + 0.0f;
+    key[i] = score_key(v);
+    stats_add(st, v);
   }
-  __syncthreads();
+  st = block_stats(st, sh);
+  Plan P = plan_stage(key, n_past, static_cast<uint32_t>(a.n_tar), static_cast<uint32_t>(n_past),
+                      st, kExcluded, hist, list_key, list_idx, sh);
+  Picker pk = make_picker(key, c0, c1, P, kExcluded, sh);
+  Stats sv{INFINITY, -INFINITY, 0u};
+  for (int i0 = c0; i0 < c1; i0 += 8) {
+    float vb[8];  // issue the VaN loads of 8 tokens before using any
+#pragma unroll
+    for (int b = 0; b < 8; ++b) vb[b] = (i0 + b < c1) ? van[i0 + b] : 0.0f;
+#pragma unroll
+    for (int b = 0; b < 8; ++b) {
+      const int i = i0 + b;
+      if (i >= c1) break;
+      if (pk.pick(key[i])) {
+        key[i] = kExcluded;
+      } else {
+        const float v = vb[b] + 0.0f;
+        key[i] = score_key(v);
+        stats_add(sv, v);
+      }
+    }
+  }
+  sv = block_stats(sv, sh);  // its barriers also publish the keys
 
-  // VaN stage over the past tokens TaR left (keys >= 1).
+  // VaN stage over the past tokens TaR left.
   const uint32_t n_rest = static_cast<uint32_t>(n_past - a.n_tar);
-  T = 0xFFFFFFFFu;
-  take = 0u;
-  cnt_eq = 0u;
-  if (a.n_van > 0)
-    find_threshold(key, n_past, static_cast<uint32_t>(a.n_van), n_rest, hist, sh, &T, &take,
-                   &cnt_eq);
-  rank = (take > 0u && take < cnt_eq) ? ties_before(key, c0, c1, T, sh) : 0u;
-  const bool all_ties_v = take >= cnt_eq;
-  for (int i = c0; i < c1; ++i) {
-    const uint32_t x = key[i];
-    if (x == kExcluded) continue;
-    bool pick = x > T && a.n_van > 0;
-    if (x == T && take > 0u) pick = all_ties_v || (rank++ < take);
-    if (pick) key[i] = kTaken;
-  }
+  P = plan_stage(key, n_past, static_cast<uint32_t>(a.n_van), n_rest, sv, kTaken, hist, list_key,
+                 list_idx, sh);
+  pk = make_picker(key, c0, c1, P, kTaken, sh);
+  for (int i = c0; i < c1; ++i)
+    if (pk.pick(key[i])) key[i] = kTaken;
   __syncthreads();
 
   // Ascending kept indices: past picks, then the recent frames.
