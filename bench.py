@@ -27,7 +27,7 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "compress-pass latency (ms) and HBM GB/s vs GB300 peak, 7B shape 6K budget"
-KERNELS = ("recent_mean", "score", "select", "gather")
+KERNELS = ("recent_mean", "score", "select", "gather", "pipeline")
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -59,8 +59,16 @@ def bytes_model(w: synth.Workload, S: int, r: int):
         "score": S * (2 * n_past * row + 8 * n_past),
         "select": S * (8 * n_past + 4 * C),
         "gather": S * (4 * C * row + 4 * C),
+        "pipeline": pass_bytes,  # the single-kernel pass does all four steps
     }
     return pass_bytes, tight, per_kernel
+
+
+def dram_min_bytes(w: synth.Workload, S: int, r: int) -> int:
+    """Least DRAM traffic any pass can have: read every K and V row once (the
+    V of recent rows is not needed), write the kept K and V rows and indices."""
+    row = w.head_dim * w.elem_bytes
+    return S * row * (2 * w.n_tokens - r * w.p + 2 * w.budget) + S * w.budget * 4
 
 
 def source_digest() -> str:
@@ -220,7 +228,7 @@ def run_gpu(args, w: synth.Workload):
     N, C, D, p = w.n_tokens, w.budget, w.head_dim, w.p
 
     ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
-             token_capacity=N)
+             token_capacity=N, single_kernel=args.single_kernel)
     r = ipv.recent_frames(w.n_frames)
     cache = PingPongCache(S, N, D, w.dtype, patch_ids=False)
     for i, st in enumerate(streams):
@@ -348,6 +356,9 @@ def run_gpu(args, w: synth.Workload):
             "per_pass_ms_p50": float(np.percentile(per_pass, 50)),
             "per_pass_ms_p99": float(np.percentile(per_pass, 99)),
             "kernel_ms": {k: round(kern_ms[k], 5) for k in KERNELS},
+            "path": "single-kernel pipeline" if args.single_kernel else "step kernels",
+            "dram_min_bytes": dram_min_bytes(w, S, r),
+            "dram_min_frac": dram_min_bytes(w, S, r) / (ms_pass_max * 1e-3) / 1e9 / peak,
             "roofline": {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": peak,
                          "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)" if peak_kind == "measured" else "fallback 6.8 TB/s",
                          "unit": "GB/s", "frac": achieved / peak, "traffic": traffic,
@@ -378,6 +389,8 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ref-slabs", type=int, default=4)
+    ap.add_argument("--single-kernel", action="store_true",
+                    help="run the pass as one persistent kernel instead of the step kernels")
     args = ap.parse_args(argv)
     w = synth.CONFIGS[args.config]
     if args.config == "stream":

@@ -69,6 +69,11 @@ typedef struct {
   int max_frame_tokens;   /* largest p = frame_grid_h*frame_grid_w (<= 65535) */
   int64_t max_slabs;      /* largest n_layers*n_kv_heads any call will use */
   int64_t token_capacity; /* rows per slab in each cache half (the slab stride) */
+  int single_kernel;      /* 0: ipv_compress runs the pass as its four step kernels
+                             (recent-frame mean, scoring, selection, compaction),
+                             one after the other; 1: as one persistent kernel whose
+                             blocks overlap the steps of different slabs. Both give
+                             bit-identical results. */
 } ipv_options;
 
 /* One tensor (K or V) of the ping-pong cache: two halves of identical
@@ -146,8 +151,9 @@ const char* ipv_status_string(ipv_status s);
 
 /* Kernel timing for benchmarks: while enabled, ipv_compress and ipv_score
  * record CUDA events around each kernel on the call's stream. Kernel ids:
- * 0 recent-frame mean, 1 scoring, 2 selection, 3 compaction. */
-#define IPV_NUM_KERNELS 4
+ * 0 recent-frame mean, 1 scoring, 2 selection, 3 compaction, 4 the
+ * single-kernel pass. */
+#define IPV_NUM_KERNELS 5
 ipv_status ipv_profile_enable(int on);
 
 /* Waits (at most timeout_ms) for the recorded events, then writes per kernel
@@ -155,6 +161,13 @@ ipv_status ipv_profile_enable(int on);
  * record. Errors: IPV_ETIMEOUT, IPV_ECUDA, IPV_EINVAL (NULL outputs). */
 ipv_status ipv_profile_collect(double ms_out[IPV_NUM_KERNELS],
                                int64_t launches_out[IPV_NUM_KERNELS], int timeout_ms);
+
+/* Diagnostic: the single-kernel pass bounds every wait and, when one runs
+ * out, sets bits in a device error word (1: a score chunk gave up waiting for
+ * its slab's recent-frame mean; 2: a block gave up waiting for work). This
+ * waits for the whole device, copies the word to *err_out (0 = no timeout
+ * since the last read) and clears it. Errors: IPV_ENOINIT, IPV_EINVAL, IPV_ECUDA. */
+ipv_status ipv_device_error(uint32_t* err_out);
 
 #ifdef __cplusplus
 }

@@ -15,7 +15,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJ = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libipv.so")
-SOURCES = ["api.cu", "score.cu", "select.cu", "gather.cu"]
+SOURCES = ["api.cu", "score.cu", "select.cu", "gather.cu", "pipeline.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 
@@ -26,7 +26,8 @@ def _stale(out: str, deps: list[str]) -> bool:
 
 def build(force: bool = False, extra_flags: list[str] | None = None, verbose: bool = False) -> str:
     os.makedirs(OBJ, exist_ok=True)
-    headers = [os.path.join(CSRC, "ipv_common.cuh"), os.path.join(INCLUDE, "ipv.h")]
+    headers = [os.path.join(CSRC, "ipv_common.cuh"), os.path.join(CSRC, "pass_device.cuh"),
+               os.path.join(INCLUDE, "ipv.h")]
     procs, objs = [], []
     for src in SOURCES:
         path = os.path.join(CSRC, src)

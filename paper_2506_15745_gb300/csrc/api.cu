@@ -10,6 +10,8 @@
 #include "ipv.h"
 #include "ipv_common.cuh"
 
+static_assert(ipv::kMaxTokens == IPV_MAX_TOKENS, "selection shared-memory limit");
+
 namespace {
 
 struct EventPair {
@@ -23,6 +25,9 @@ struct State {
   float* tar = nullptr;   // [max_slabs][token_capacity]
   float* van = nullptr;
   float* m = nullptr;     // [max_slabs][max_frame_tokens][max_head_dim]
+  ipv::PipeState* pstate = nullptr;
+  unsigned* pflags = nullptr;  // [kPipeFlags][max_slabs]
+  bool pipe_dirty = false;     // a failed launch may have left queue state behind
   bool profiling = false;
   std::vector<EventPair> pool;                      // idle event pairs
   std::vector<EventPair> pending[IPV_NUM_KERNELS];  // recorded, not yet read
@@ -200,6 +205,8 @@ void ipv_shutdown(void) {
   cudaFree(g.tar);
   cudaFree(g.van);
   cudaFree(g.m);
+  cudaFree(g.pstate);
+  cudaFree(g.pflags);
   g = State{};
 }
 
@@ -214,6 +221,8 @@ ipv_status ipv_init(const ipv_options* opt) {
   if (opt->max_slabs <= 0 || opt->max_slabs > INT32_MAX) return fail(IPV_EINVAL, "max_slabs must be in [1, 2^31)");
   if (opt->token_capacity <= 0 || opt->token_capacity > INT32_MAX)
     return fail(IPV_EINVAL, "token_capacity must be in [1, 2^31)");
+  if (opt->single_kernel != 0 && opt->single_kernel != 1)
+    return fail(IPV_EINVAL, "single_kernel must be 0 or 1");
   ipv_shutdown();
   int n_dev = 0;
   cudaError_t e = cudaGetDeviceCount(&n_dev);
@@ -226,19 +235,34 @@ ipv_status ipv_init(const ipv_options* opt) {
   if ((e = ipv::score_prepare(opt->max_frame_tokens, opt->max_head_dim)) != cudaSuccess)
     return cuda_fail(e, "no usable kernel image for this device (built for sm_103a)");
   if ((e = ipv::select_prepare(IPV_MAX_TOKENS)) != cudaSuccess) return cuda_fail(e, "select kernel set-up");
+  if ((e = ipv::pipeline_prepare()) != cudaSuccess) return cuda_fail(e, "pipeline kernel set-up");
   State s;
   s.opt = *opt;
   s.num_sms = prop.multiProcessorCount;
   const size_t score_bytes = static_cast<size_t>(opt->max_slabs) * opt->token_capacity * sizeof(float);
   const size_t m_bytes =
       static_cast<size_t>(opt->max_slabs) * opt->max_frame_tokens * opt->max_head_dim * sizeof(float);
+  const size_t flag_bytes = ipv::kPipeFlags * static_cast<size_t>(opt->max_slabs) * sizeof(unsigned);
   if (cudaMalloc(&s.tar, score_bytes) != cudaSuccess || cudaMalloc(&s.van, score_bytes) != cudaSuccess ||
-      cudaMalloc(&s.m, m_bytes) != cudaSuccess) {
+      cudaMalloc(&s.m, m_bytes) != cudaSuccess ||
+      cudaMalloc(&s.pstate, sizeof(ipv::PipeState)) != cudaSuccess ||
+      cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess) {
     cudaGetLastError();
     cudaFree(s.tar);
     cudaFree(s.van);
     cudaFree(s.m);
+    cudaFree(s.pstate);
+    cudaFree(s.pflags);
     return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated", 2 * score_bytes + m_bytes);
+  }
+  if ((e = cudaMemset(s.pstate, 0, sizeof(ipv::PipeState))) != cudaSuccess ||
+      (e = cudaMemset(s.pflags, 0, flag_bytes)) != cudaSuccess) {
+    cudaFree(s.tar);
+    cudaFree(s.van);
+    cudaFree(s.m);
+    cudaFree(s.pstate);
+    cudaFree(s.pflags);
+    return cuda_fail(e, "clearing the pipeline state");
   }
   s.ready = true;
   g = s;
@@ -281,6 +305,7 @@ ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_he
   a.van = van_out;
   a.zero_recent = 1;
   a.num_sms = g.num_sms;
+  a.error = &g.pstate->error;
   prof_begin(0, st);
   cudaError_t e = ipv::launch_recent_mean(a, st);
   prof_end(0, st);
@@ -365,14 +390,7 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   a.van = g.van;
   a.zero_recent = 0;
   a.num_sms = g.num_sms;
-  prof_begin(0, st);
-  cudaError_t e = ipv::launch_recent_mean(a, st);
-  prof_end(0, st);
-  if (e != cudaSuccess) return cuda_fail(e, "recent-frame mean kernel");
-  prof_begin(1, st);
-  e = ipv::launch_score(a, st);
-  prof_end(1, st);
-  if (e != cudaSuccess) return cuda_fail(e, "scoring kernel");
+  a.error = &g.pstate->error;
 
   ipv::SelectArgs sa{};
   sa.tar = g.tar;
@@ -383,10 +401,6 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   sa.budget = budget;
   split_budget(budget, tar_ratio, sh.rp, &sa.n_tar, &sa.n_van);
   sa.kept = kept_idx_out;
-  prof_begin(2, st);
-  e = ipv::launch_select(sa, st);
-  prof_end(2, st);
-  if (e != cudaSuccess) return cuda_fail(e, "selection kernel");
 
   ipv::GatherArgs ga{};
   ga.k_src = k->buf[k->cur];
@@ -402,12 +416,83 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   ga.row_bytes = sh.D * elem_bytes();
   ga.p = sh.p;
   ga.num_sms = g.num_sms;
+
+  cudaError_t e;
+  if (g.opt.single_kernel) {
+    if (g.pipe_dirty) {
+      if ((e = cudaMemsetAsync(g.pstate, 0, sizeof(ipv::PipeState), st)) != cudaSuccess ||
+          (e = cudaMemsetAsync(g.pflags, 0, ipv::kPipeFlags * sh.S * sizeof(unsigned), st)) != cudaSuccess)
+        return cuda_fail(e, "clearing the pipeline state");
+      g.pipe_dirty = false;
+    }
+    ipv::PipeArgs pa{};
+    pa.sc = a;
+    pa.se = sa;
+    pa.ga = ga;
+    pa.state = g.pstate;
+    pa.flags = g.pflags;
+    const int64_t n_past = sh.N - sh.rp;
+    pa.n_sc = static_cast<int>((n_past + 1023) / 1024);
+    pa.rows_sc = static_cast<int>((n_past + pa.n_sc - 1) / pa.n_sc);
+    pa.n_ga = static_cast<int>((budget + 1023) / 1024);
+    pa.rows_ga = static_cast<int>((budget + pa.n_ga - 1) / pa.n_ga);
+    pa.group = 4;
+    pa.lead = 2;
+    pa.n_groups = static_cast<int>((sh.S + pa.group - 1) / pa.group);
+    pa.spin_limit = int64_t{1} << 20;
+    pa.nst = ipv::pipeline_stages(sh.p, sh.D, elem_bytes());
+    // The selection needs its keys in shared memory as well (one item at a time).
+    if (ipv::pipeline_smem_bytes(sh.N - sh.rp) > ipv::kBulkSmemMax)
+      return fail(IPV_EINVAL, "n_tokens %lld too large for the single-kernel pass", static_cast<long long>(sh.N));
+    prof_begin(4, st);
+    e = ipv::launch_pipeline(pa, g.num_sms, st);
+    prof_end(4, st);
+    if (e != cudaSuccess) {
+      g.pipe_dirty = true;
+      return cuda_fail(e, "single-kernel pass");
+    }
+    k->cur = 1 - k->cur;
+    v->cur = 1 - v->cur;
+    return IPV_OK;
+  }
+
+  prof_begin(0, st);
+  e = ipv::launch_recent_mean(a, st);
+  prof_end(0, st);
+  if (e != cudaSuccess) return cuda_fail(e, "recent-frame mean kernel");
+  prof_begin(1, st);
+  e = ipv::launch_score(a, st);
+  prof_end(1, st);
+  if (e != cudaSuccess) return cuda_fail(e, "scoring kernel");
+  prof_begin(2, st);
+  e = ipv::launch_select(sa, st);
+  prof_end(2, st);
+  if (e != cudaSuccess) return cuda_fail(e, "selection kernel");
+
   prof_begin(3, st);
   e = ipv::launch_gather(ga, st);
   prof_end(3, st);
   if (e != cudaSuccess) return cuda_fail(e, "compaction kernel");
   k->cur = 1 - k->cur;
   v->cur = 1 - v->cur;
+  return IPV_OK;
+}
+
+ipv_status ipv_device_error(uint32_t* err_out) {
+  if (!err_out) return fail(IPV_EINVAL, "err_out must not be NULL");
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  cudaSetDevice(g.opt.device);
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  ipv::PipeState ps;
+  if ((e = cudaMemcpy(&ps, g.pstate, sizeof ps, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "reading the pipeline state");
+  *err_out = ps.error;
+  if (ps.error != 0u) {
+    ps.error = 0u;
+    if ((e = cudaMemcpy(g.pstate, &ps, sizeof ps, cudaMemcpyHostToDevice)) != cudaSuccess)
+      return cuda_fail(e, "clearing the pipeline error");
+  }
   return IPV_OK;
 }
 

@@ -9,70 +9,17 @@
 // and the matching V row; the flattened (slab, j) space is strided over the
 // whole grid with several rows in flight per half-warp. Patch ids travel with
 // their rows.
-#include "ipv_common.cuh"
+#include "pass_device.cuh"
 
 namespace ipv {
 namespace {
 
 template <int CPL>
 __global__ void __launch_bounds__(512, 2) gather_kernel(GatherArgs a) {
-  constexpr int kUnroll = CPL >= 4 ? 1 : 4 / CPL;
-  const int lane = threadIdx.x & 15;
+  constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
   const int64_t n_hw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
   const int64_t hw = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 4;
-  const int64_t total = a.n_slabs * a.budget;
-  const int n_chunks = a.row_bytes / 16;
-  const char* ks = static_cast<const char*>(a.k_src);
-  const char* vs = static_cast<const char*>(a.v_src);
-  char* kd = static_cast<char*>(a.k_dst);
-  char* vd = static_cast<char*>(a.v_dst);
-
-  for (int64_t g0 = hw; g0 < total; g0 += n_hw * kUnroll) {
-    uint4 kr[kUnroll][CPL], vr[kUnroll][CPL];
-    int64_t dst_off[kUnroll];
-    int src_n[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t g = g0 + u * n_hw;
-      int n = -1;
-      int64_t s = 0, j = 0;
-      if (g < total) {
-        s = g / a.budget;
-        j = g - s * a.budget;
-        n = a.kept[g];
-        if (n >= a.cap) n = -1;  // never produced by the selection; ignore
-      }
-      src_n[u] = n;
-      dst_off[u] = (s * a.cap + j) * a.row_bytes;
-      const int64_t src_off = (s * a.cap + (n < 0 ? 0 : n)) * a.row_bytes;
-#pragma unroll
-      for (int c = 0; c < CPL; ++c) {
-        const int ch = lane + 16 * c;
-        const bool ld = n >= 0 && ch < n_chunks;
-        kr[u][c] = ld ? ld_stream(ks + src_off + ch * 16) : make_uint4(0, 0, 0, 0);
-        vr[u][c] = ld ? ld_stream(vs + src_off + ch * 16) : make_uint4(0, 0, 0, 0);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      if (src_n[u] < 0) continue;
-#pragma unroll
-      for (int c = 0; c < CPL; ++c) {
-        const int ch = lane + 16 * c;
-        if (ch < n_chunks) {
-          st_stream(kd + dst_off[u] + ch * 16, kr[u][c]);
-          st_stream(vd + dst_off[u] + ch * 16, vr[u][c]);
-        }
-      }
-      if (a.pid_dst && lane == 0) {
-        const int64_t g = g0 + u * n_hw;
-        const int64_t s = g / a.budget;
-        const int64_t j = g - s * a.budget;
-        a.pid_dst[s * a.cap + j] = a.pid_src ? a.pid_src[s * a.cap + src_n[u]]
-                                             : static_cast<uint16_t>(src_n[u] % a.p);
-      }
-    }
-  }
+  dev::gather_range<CPL, kU>(a, 0, a.n_slabs * a.budget, hw, n_hw);
 }
 
 template <int CPL>
@@ -87,10 +34,13 @@ cudaError_t dispatch(const GatherArgs& a, cudaStream_t st) {
 
 }  // namespace
 
+int gather_cpl(int row_bytes) {
+  const int n_chunks = row_bytes / 16;
+  return n_chunks <= 16 ? 1 : n_chunks <= 32 ? 2 : n_chunks <= 64 ? 4 : 8;
+}
+
 cudaError_t launch_gather(const GatherArgs& a, cudaStream_t st) {
-  const int n_chunks = a.row_bytes / 16;
-  const int cpl = n_chunks <= 16 ? 1 : n_chunks <= 32 ? 2 : n_chunks <= 64 ? 4 : 8;
-  switch (cpl) {
+  switch (gather_cpl(a.row_bytes)) {
     case 1: return dispatch<1>(a, st);
     case 2: return dispatch<2>(a, st);
     case 4: return dispatch<4>(a, st);

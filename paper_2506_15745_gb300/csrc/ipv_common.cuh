@@ -10,6 +10,7 @@ namespace ipv {
 constexpr float kNormEps = 1e-12f;   // cos(a,b) = a.b / (max|a|,eps)(max|b|,eps)
 constexpr int kSelectThreads = 1024;
 constexpr int kSelectBins = 2048;
+constexpr int64_t kMaxTokens = 49152;  // IPV_MAX_TOKENS: selection keys live in shared memory
 
 // ---------------------------------------------------------------- device helpers
 // 16-byte global load that bypasses L1 (each cache row is read once per
@@ -27,6 +28,60 @@ __device__ __forceinline__ void st_stream(void* p, uint4 v) {
   asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
                "r"(v.w)
                : "memory");
+}
+
+// ---------------------------------------------------------------- bulk copies
+// 1-D bulk copies (cp.async.bulk, the TMA engine) from global into shared
+// memory, completed on an mbarrier that also counts the bytes. Addresses and
+// sizes are multiples of 16 bytes.
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+// Makes barrier initialisation visible to the bulk-copy (async) proxy.
+__device__ __forceinline__ void mbar_init_fence() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0u;
+}
+
+// Orders this thread's earlier generic-proxy shared-memory accesses before
+// its later bulk copies into shared memory.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Bounded wait for a barrier phase; false if it did not complete in time.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (int it = 0; it < (1 << 22); ++it)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
 }
 
 // Elements held by one 16-byte chunk, widened to fp32.
@@ -82,8 +137,18 @@ struct ScoreArgs {
   float* van;
   int zero_recent;          // write 0 to the recent-frame entries of tar/van
   int num_sms;
+  unsigned* error;          // device word: bit 2 set if a bulk-copy wait timed out
 };
 
+int row_shape(int D, int is_bf16);  // encoded (lanes per row, chunks per lane)
+// Bulk-copy-fed scoring: shape code (lanes per row * 10 + chunks per lane,
+// 324 for 32 lanes x 4), shared memory for the m table plus an nst-stage
+// ring, and the deepest ring (<= kMaxStages, >= 2) that fits (0: none).
+constexpr int kMaxStages = 4;
+constexpr size_t kBulkSmemMax = 226 * 1024;  // 227 KB per block, less room for static shared memory
+int bulk_shape(int D, int is_bf16);
+size_t bulk_smem_bytes(int p, int D, int elem, int nst, int threads);
+int bulk_stages(int p, int D, int elem, int threads);
 cudaError_t launch_recent_mean(const ScoreArgs& a, cudaStream_t st);
 cudaError_t launch_score(const ScoreArgs& a, cudaStream_t st);
 size_t score_smem_bytes(int p, int D);
@@ -100,7 +165,7 @@ struct SelectArgs {
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
 cudaError_t launch_passthrough(int32_t* kept, int64_t n_slabs, int64_t n_tokens, int64_t budget,
                                cudaStream_t st);
-size_t select_smem_bytes(int64_t n_tokens);
+size_t select_smem_bytes(int64_t n_past);
 cudaError_t select_prepare(int64_t max_tokens);
 
 struct GatherArgs {
@@ -116,6 +181,37 @@ struct GatherArgs {
   int num_sms;
 };
 
+int gather_cpl(int row_bytes);  // 16-byte chunks per lane of a half-warp row copy
 cudaError_t launch_gather(const GatherArgs& a, cudaStream_t st);
+
+// Single-kernel pass (pipeline.cu). The queue state lives in library scratch,
+// is zero before a launch and is reset by the kernel's last block.
+struct PipeState {
+  unsigned main_head;  // next main-queue ticket
+  unsigned sel_low;    // slabs below have their selection taken
+  unsigned gat_low;    // slabs below have all gather chunks handed out
+  unsigned exited;     // blocks that have left
+  unsigned error;      // bit 0: a score item's wait timed out; bit 1: an idle wait timed out
+  unsigned pad[3];
+};
+constexpr int kPipeFlags = 5;  // per-slab words: mean, scores, select claim, select done, gather ticket
+
+struct PipeArgs {
+  ScoreArgs sc;      // tar/van/m point at library scratch
+  SelectArgs se;
+  GatherArgs ga;
+  PipeState* state;
+  unsigned* flags;   // [kPipeFlags][n_slabs]
+  int n_sc, rows_sc; // score chunks per slab, past rows per chunk
+  int n_ga, rows_ga; // gather chunks per slab, kept rows per chunk
+  int group, lead, n_groups;
+  int nst;           // bulk-copy stages for score chunks (0: 16-byte loads)
+  int64_t spin_limit;
+};
+
+size_t pipeline_smem_bytes(int64_t n_past);
+int pipeline_stages(int p, int D, int elem);  // bulk-copy stages that fit (0: none)
+cudaError_t pipeline_prepare();
+cudaError_t launch_pipeline(const PipeArgs& a, int num_sms, cudaStream_t st);
 
 }  // namespace ipv

@@ -15,8 +15,8 @@ LIB_PATH = os.path.join(_HERE, "libipv.so")
 
 IPV_OK, IPV_EINVAL, IPV_ENOINIT, IPV_ENOMEM, IPV_ECUDA, IPV_ETIMEOUT = range(6)
 IPV_BF16, IPV_F32 = 0, 1
-NUM_KERNELS = 4
-KERNEL_NAMES = ("recent_mean", "score", "select", "gather")
+NUM_KERNELS = 5
+KERNEL_NAMES = ("recent_mean", "score", "select", "gather", "pipeline")
 MAX_TOKENS = 49152
 
 
@@ -30,7 +30,7 @@ class Options(ctypes.Structure):
     _fields_ = [("device", ctypes.c_int), ("dtype", ctypes.c_int),
                 ("recent_frames", ctypes.c_int), ("max_head_dim", ctypes.c_int),
                 ("max_frame_tokens", ctypes.c_int), ("max_slabs", ctypes.c_int64),
-                ("token_capacity", ctypes.c_int64)]
+                ("token_capacity", ctypes.c_int64), ("single_kernel", ctypes.c_int)]
 
 
 class KV(ctypes.Structure):
@@ -84,8 +84,9 @@ def load():
         lib.ipv_profile_enable.argtypes = [I32]
         lib.ipv_profile_collect.argtypes = [ctypes.POINTER(ctypes.c_double),
                                             ctypes.POINTER(ctypes.c_int64), I32]
+        lib.ipv_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32)]
         for name in ("ipv_init", "ipv_compress", "ipv_score", "ipv_select",
-                     "ipv_profile_enable", "ipv_profile_collect"):
+                     "ipv_profile_enable", "ipv_profile_collect", "ipv_device_error"):
             getattr(lib, name).restype = I32
         _lib = lib
     return _lib
@@ -108,9 +109,10 @@ def last_error() -> str:
 
 
 def init(*, device: int = 0, dtype: str = "bf16", recent_frames: int = 0, max_head_dim: int,
-         max_frame_tokens: int, max_slabs: int, token_capacity: int) -> None:
+         max_frame_tokens: int, max_slabs: int, token_capacity: int,
+         single_kernel: bool = False) -> None:
     opt = Options(device, IPV_BF16 if dtype == "bf16" else IPV_F32, recent_frames, max_head_dim,
-                  max_frame_tokens, max_slabs, token_capacity)
+                  max_frame_tokens, max_slabs, token_capacity, int(bool(single_kernel)))
     _check(load().ipv_init(ctypes.byref(opt)))
 
 
@@ -142,6 +144,13 @@ def select(tar, van, n_slabs: int, n_tokens: int, frame_grid_h: int, frame_grid_
            budget: int, tar_ratio: float, kept_idx_out, stream=None) -> None:
     _check(load().ipv_select(_ptr(tar), _ptr(van), n_slabs, n_tokens, frame_grid_h, frame_grid_w,
                              budget, tar_ratio, _ptr(kept_idx_out), _stream(stream)))
+
+
+def device_error() -> int:
+    """Timeout bits of the single-kernel pass since the last read (waits for the device)."""
+    out = ctypes.c_uint32(0)
+    _check(load().ipv_device_error(ctypes.byref(out)))
+    return out.value
 
 
 def profile_enable(on: bool) -> None:

@@ -39,9 +39,9 @@ def _shutdown_after():
     ipv.shutdown()
 
 
-def init_for(S, cap, D, p, dtype, recent_frames=0):
+def init_for(S, cap, D, p, dtype, recent_frames=0, single_kernel=False):
     ipv.init(device=0, dtype=dtype, recent_frames=recent_frames, max_head_dim=D,
-             max_frame_tokens=p, max_slabs=S, token_capacity=cap)
+             max_frame_tokens=p, max_slabs=S, token_capacity=cap, single_kernel=single_kernel)
 
 
 def check_pass(cache, L, H, N, gh, gw, budget, alpha, pid_valid, slabs=None):
@@ -316,3 +316,90 @@ def test_large_config_sampled():
     finally:
         del cache
         torch.cuda.empty_cache()
+
+
+def _run_both(w, L, make_cache, pid_valid, passes=1):
+    """Run `passes` passes with the single-kernel pipeline and with the staged
+    kernels on identical inputs; return both (kept, cache) results."""
+    out = []
+    for single in (True, False):
+        init_for(w_slabs(w, L), w.n_tokens, w.head_dim, w.p, w.dtype, single_kernel=single)
+        cache = make_cache()
+        kept = torch.empty((cache.n_slabs, w.budget), dtype=torch.int32, device="cuda")
+        for _ in range(passes):
+            cache.n_tokens = w.n_tokens
+            cache.compress(L, w.n_kv_heads, w.grid_h, w.grid_w, w.budget, w.tar_ratio, kept,
+                           pid_valid=pid_valid)
+        torch.cuda.synchronize()
+        assert ipv.device_error() == 0
+        out.append((kept.clone(), cache))
+        ipv.shutdown()
+    return out
+
+
+def w_slabs(w, L):
+    return L * w.n_kv_heads
+
+
+@pytest.mark.parametrize("name", ["llava", "qwen", "tiny"])
+def test_pipeline_matches_staged(name):
+    """The single-kernel pass and the four step kernels run the same device
+    arithmetic: indices, compacted rows and patch ids are bit-identical."""
+    w = synth.CONFIGS[name]
+    L = w.n_layers
+
+    def make_cache():
+        c = PingPongCache(w.slabs_per_stream, w.n_tokens, w.head_dim, w.dtype, patch_ids=True)
+        if w.dtype == "f32":
+            K, V = synth.host_generate(w)
+            c.k[0] = to_dev(K, w.dtype)
+            c.v[0] = to_dev(V, w.dtype)
+        else:
+            synth.device_generate(w, c.k[0], c.v[0])
+        return c
+
+    (kp, cp), (ks, cs) = _run_both(w, L, make_cache, pid_valid=False)
+    B = w.budget
+    assert torch.equal(kp, ks)
+    assert cp.cur == cs.cur == 1
+    assert torch.equal(cp.k[1, :, :B], cs.k[1, :, :B])
+    assert torch.equal(cp.v[1, :, :B], cs.v[1, :, :B])
+    assert torch.equal(cp.pid[1, :, :B], cs.pid[1, :, :B])
+
+
+def test_pipeline_repeated_passes_and_patch_ids():
+    """Back-to-back single-kernel passes reuse the queue state the previous
+    pass reset; with shuffled patch ids the result still equals the staged path."""
+    S, f, gh, gw, D = 24, 16, 7, 7, 128
+    w = synth.Workload("case", 1, S, D, "bf16", gh, gw, f, 500, 0.5, seed=21)
+    p, N = w.p, w.n_tokens
+    K, V = synth.host_generate(w)
+    r = oracle.recent_frames(f)
+    n_past = N - r * p
+    perm = np.random.default_rng(4).permutation(n_past)
+    K[:, :n_past], V[:, :n_past] = K[:, perm], V[:, perm]
+    pid = np.tile((np.arange(N) % p).astype(np.uint16), (S, 1))
+    pid[:, :n_past] = (perm % p).astype(np.uint16)
+
+    def make_cache():
+        c = PingPongCache(S, N, D, "bf16", patch_ids=True)
+        c.k[0] = to_dev(K, "bf16")
+        c.v[0] = to_dev(V, "bf16")
+        c.pid[0] = torch.from_numpy(pid.view(np.int16)).cuda()
+        return c
+
+    results = []
+    for single in (True, False):
+        init_for(S, N, D, p, "bf16", single_kernel=single)
+        kept = torch.empty((S, w.budget), dtype=torch.int32, device="cuda")
+        c = make_cache()
+        for _ in range(5):  # identical input each time: cur reset to the source half
+            k_s, v_s = c.structs(pid_valid=True)
+            k_s.cur = v_s.cur = 0
+            ipv.compress(k_s, v_s, 1, S, D, N, gh, gw, w.budget, w.tar_ratio, kept)
+        torch.cuda.synchronize()
+        assert ipv.device_error() == 0
+        results.append((kept.clone(), c.k[1, :, :w.budget].clone(), c.pid[1, :, :w.budget].clone()))
+        ipv.shutdown()
+    for a, b in zip(*results):
+        assert torch.equal(a, b)
