@@ -162,6 +162,33 @@ ipv_status ipv_profile_enable(int on);
 ipv_status ipv_profile_collect(double ms_out[IPV_NUM_KERNELS],
                                int64_t launches_out[IPV_NUM_KERNELS], int timeout_ms);
 
+/* ipv_compress without any device allocation, for callers that cannot
+ * allocate device memory: a process whose device memory belongs to a caching
+ * allocator or to a fixed budget the library must not grow, or code on a path
+ * where cudaMalloc/cudaFree (which can synchronise the device) are not allowed.
+ * The paper has no counterpart; this is a deployment variant of the same pass.
+ *
+ * Same arguments, layout and results as ipv_compress, except that the options
+ * of ipv_init (element type, slab stride token_capacity, recent_frames; 0 =
+ * default r) are passed in, and no ipv_init is needed. Runs on the current
+ * device. The kernels' working memory (TaR and VaN of every token, fp32
+ * [n_slabs][n_tokens] each, and the recent-frame mean of every patch, fp32
+ * [n_slabs][p][head_dim], each rounded up to 256 bytes) comes from one
+ * statically sized array of IPV_STATIC_SCRATCH_BYTES in the library's device
+ * image, held on every device that loads the library until the process exits.
+ * A pass that needs more is rejected with IPV_EINVAL before anything is
+ * enqueued (the LLaVA-OV-7B and Qwen2-VL-7B shapes fit).
+ * The first call on a device sets that device up once (kernel limits and
+ * cudaGetSymbolAddress of the array): make it before any stream capture. All
+ * calls on a device share the array, so calls that may overlap on the GPU
+ * race and must be ordered by the caller. Errors: as ipv_compress, plus
+ * IPV_EINVAL for a pass too large for the array. */
+#define IPV_STATIC_SCRATCH_BYTES (32u << 20)
+ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype, int64_t token_capacity,
+                               int recent_frames, int n_layers, int n_kv_heads, int head_dim,
+                               int64_t n_tokens, int frame_grid_h, int frame_grid_w, int64_t budget,
+                               float tar_ratio, int32_t* kept_idx_out, void* stream);
+
 /* Diagnostic: the single-kernel pass bounds every wait and, when one runs
  * out, sets bits in a device error word (1: a score chunk gave up waiting for
  * its slab's recent-frame mean; 2: a block gave up waiting for work). This

@@ -181,6 +181,11 @@ ipv_status after_launch(cudaError_t e, const char* what) {
 
 }  // namespace
 
+namespace ipv {
+// Lets other translation units of the library report through ipv_last_error.
+void record_error(ipv_status s, const char* msg) { fail(s, "%s", msg); }
+}  // namespace ipv
+
 extern "C" {
 
 const char* ipv_status_string(ipv_status s) {

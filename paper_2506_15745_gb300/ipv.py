@@ -85,8 +85,11 @@ def load():
         lib.ipv_profile_collect.argtypes = [ctypes.POINTER(ctypes.c_double),
                                             ctypes.POINTER(ctypes.c_int64), I32]
         lib.ipv_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32)]
+        lib.ipv_compress_static.argtypes = [KVP, KVP, I32, I64, I32, I32, I32, I32, I64, I32, I32,
+                                            I64, F, P, P]
         for name in ("ipv_init", "ipv_compress", "ipv_score", "ipv_select",
-                     "ipv_profile_enable", "ipv_profile_collect", "ipv_device_error"):
+                     "ipv_profile_enable", "ipv_profile_collect", "ipv_device_error",
+                     "ipv_compress_static"):
             getattr(lib, name).restype = I32
         _lib = lib
     return _lib
@@ -131,6 +134,22 @@ def compress(k: KV, v: KV, n_layers: int, n_kv_heads: int, head_dim: int, n_toke
     _check(load().ipv_compress(ctypes.byref(k), ctypes.byref(v), n_layers, n_kv_heads, head_dim,
                                n_tokens, frame_grid_h, frame_grid_w, budget, tar_ratio,
                                _ptr(kept_idx_out), _stream(stream)))
+
+
+STATIC_SCRATCH_BYTES = 32 << 20
+
+
+def compress_static(k: KV, v: KV, dtype: str, token_capacity: int, recent_frames: int,
+                    n_layers: int, n_kv_heads: int, head_dim: int, n_tokens: int,
+                    frame_grid_h: int, frame_grid_w: int, budget: int, tar_ratio: float,
+                    kept_idx_out, stream=None) -> None:
+    """ipv_compress_static: the pass with no device allocation and no ipv_init
+    (its working memory is a fixed array in the library's device image)."""
+    _check(load().ipv_compress_static(ctypes.byref(k), ctypes.byref(v),
+                                      IPV_BF16 if dtype == "bf16" else IPV_F32, token_capacity,
+                                      recent_frames, n_layers, n_kv_heads, head_dim, n_tokens,
+                                      frame_grid_h, frame_grid_w, budget, tar_ratio,
+                                      _ptr(kept_idx_out), _stream(stream)))
 
 
 def score(k: KV, v: KV, n_layers: int, n_kv_heads: int, head_dim: int, n_tokens: int,
