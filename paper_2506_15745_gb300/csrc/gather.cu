@@ -16,6 +16,8 @@ namespace {
 
 template <int CPL>
 __global__ void __launch_bounds__(512, 2) gather_kernel(GatherArgs a) {
+  pdl_trigger();
+  pdl_wait();  // the kept indices come from the selection kernel
   constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
   const int64_t n_hw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
   const int64_t hw = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 4;
@@ -28,8 +30,7 @@ cudaError_t dispatch(const GatherArgs& a, cudaStream_t st) {
   cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gather_kernel<CPL>, 512, 0);
   if (e != cudaSuccess) return e;
   per_sm = per_sm < 1 ? 1 : per_sm;
-  gather_kernel<CPL><<<a.num_sms * per_sm, 512, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch(gather_kernel<CPL>, a.num_sms * per_sm, 512, 0, st, true, a);
 }
 
 }  // namespace

@@ -30,6 +30,32 @@ __device__ __forceinline__ void st_stream(void* p, uint4 v) {
                : "memory");
 }
 
+// ---------------------------------------------------------------- dependent launch
+// Programmatic dependent launch: a kernel lets the next kernel of the stream
+// start its blocks as soon as every block of this one has started (trigger),
+// and a kernel waits for the previous kernel's completion and memory before
+// reading its results (wait). Without the launch attribute both are no-ops.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Launches kernel on st; with pdl the launch may overlap the previous kernel
+// of the stream, which the kernel must then wait for with pdl_wait().
+template <typename... Params, typename... Args>
+cudaError_t launch(void (*kernel)(Params...), unsigned grid, unsigned block, size_t smem,
+                   cudaStream_t st, bool pdl, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // ---------------------------------------------------------------- bulk copies
 // 1-D bulk copies (cp.async.bulk, the TMA engine) from global into shared
 // memory, completed on an mbarrier that also counts the bytes. Addresses and

@@ -22,6 +22,7 @@ constexpr int kScoreThreads = 768;
 // m_q for 32/LPR patches per warp, patches flattened over (slab, q).
 template <typename T, int LPR, int CPL>
 __global__ void __launch_bounds__(128) recent_mean_kernel(ScoreArgs a) {
+  pdl_trigger();
   constexpr int RPW = 32 / LPR;
   const int grp = (threadIdx.x & 31) / LPR;
   const int64_t warp = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
@@ -38,6 +39,8 @@ __global__ void __launch_bounds__(128) recent_mean_kernel(ScoreArgs a) {
 // (SMEM_M), or read through L1/L2.
 template <typename T, int LPR, int CPL, bool SMEM_M>
 __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(ScoreArgs a) {
+  pdl_trigger();
+  pdl_wait();  // m comes from the recent-frame mean kernel
   constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
   extern __shared__ float4 sm_m4[];
   const int lane = threadIdx.x & 31;
@@ -82,13 +85,15 @@ cudaError_t dispatch_score(const ScoreArgs& a, cudaStream_t st) {
                                                       kScoreThreads, smem);
     if (e != cudaSuccess) return e;
     per_sm = per_sm < 1 ? 1 : per_sm;
-    score_kernel<T, LPR, CPL, true><<<a.num_sms * per_sm, kScoreThreads, smem, st>>>(a);
+    e = launch(score_kernel<T, LPR, CPL, true>, a.num_sms * per_sm, kScoreThreads, smem, st, true, a);
+    if (e != cudaSuccess) return e;
   } else {
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_kernel<T, LPR, CPL, false>,
                                                       kScoreThreads, 0);
     if (e != cudaSuccess) return e;
     per_sm = per_sm < 1 ? 1 : per_sm;
-    score_kernel<T, LPR, CPL, false><<<a.num_sms * per_sm, kScoreThreads, 0, st>>>(a);
+    e = launch(score_kernel<T, LPR, CPL, false>, a.num_sms * per_sm, kScoreThreads, 0, st, true, a);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }

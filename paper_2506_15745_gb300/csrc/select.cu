@@ -9,6 +9,8 @@ namespace {
 __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a) {
   extern __shared__ uint32_t sm_sel[];
   __shared__ dev::SelShared sh;
+  pdl_trigger();
+  pdl_wait();  // the scores come from the scoring kernel
   dev::select_slab<kSelectThreads>(a, blockIdx.x, sm_sel, sh);
 }
 
@@ -35,8 +37,7 @@ cudaError_t select_prepare(int64_t max_tokens) {
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st) {
   const size_t smem = select_smem_bytes(a.n_tokens - a.rp);
-  select_kernel<<<static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch(select_kernel, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st, true, a);
 }
 
 cudaError_t launch_passthrough(int32_t* kept, int64_t n_slabs, int64_t n_tokens, int64_t budget,
