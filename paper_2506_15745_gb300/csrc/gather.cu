@@ -21,7 +21,7 @@ __global__ void __launch_bounds__(512, 2) gather_kernel(GatherArgs a) {
   constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
   const int64_t n_hw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
   const int64_t hw = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 4;
-  dev::gather_range<CPL, kU>(a, 0, a.n_slabs * a.budget, hw, n_hw);
+  dev::gather_range<CPL, kU, true>(a, 0, a.n_slabs * a.budget, hw, n_hw);
 }
 
 template <int CPL>

@@ -17,7 +17,7 @@ constexpr int64_t kMaxTokens = 49152;  // IPV_MAX_TOKENS: selection keys live in
 // kernel). Only for data no thread writes while the kernel runs.
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
   uint4 r;
-  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
                : "l"(p));
   return r;
@@ -103,6 +103,12 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// Asks the bulk-copy engine to bring [p, p + bytes) into L2 (no data is
+// returned; bytes a multiple of 16, p 16-byte aligned).
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 // Bounded wait for a barrier phase; false if it did not complete in time.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   for (int it = 0; it < (1 << 22); ++it)
@@ -183,6 +189,10 @@ cudaError_t score_prepare(int max_p, int max_D);
 struct SelectArgs {
   const float* tar;   // [S][n_tokens]
   const float* van;
+  const void* k_pf;   // if set: K/V halves whose recent rows are prefetched into L2
+  const void* v_pf;   // for the compaction that follows ([S][cap][row_bytes])
+  int64_t cap_pf;
+  int row_bytes_pf;
   int64_t n_slabs, n_tokens;
   int64_t rp, n_tar, n_van, budget;
   int32_t* kept;      // [S][budget]

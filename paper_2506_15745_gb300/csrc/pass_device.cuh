@@ -808,7 +808,7 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
 // ... of the flattened (slab, j) range [g_begin, g_end), kU rows in flight.
 // Kept indices and source patch ids are read with plain loads (the kept
 // indices may have been written earlier in the same kernel).
-template <int CPL, int kU>
+template <int CPL, int kU, bool REVERSE = false>
 __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begin, int64_t g_end,
                                              int64_t hw, int64_t n_hw) {
   const int lane = threadIdx.x & 15;
@@ -818,16 +818,19 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
   char* kd = static_cast<char*>(a.k_dst);
   char* vd = static_cast<char*>(a.v_dst);
 
+  // REVERSE walks the range from its end, so each slab's last rows (its
+  // recent frames, which the selection prefetches into L2) come first.
   for (int64_t g0 = g_begin + hw; g0 < g_end; g0 += n_hw * kU) {
     uint4 kr[kU][CPL], vr[kU][CPL];
     int64_t dst_off[kU];
     int src_n[kU];
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
-      const int64_t g = g0 + u * n_hw;
+      const int64_t t = g0 + u * n_hw;
+      const int64_t g = REVERSE ? g_end - 1 - (t - g_begin) : t;
       int n = -1;
       int64_t s = 0, j = 0;
-      if (g < g_end) {
+      if (t < g_end) {
         s = g / a.budget;
         j = g - s * a.budget;
         n = a.kept[g];
@@ -856,7 +859,8 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
         }
       }
       if (a.pid_dst && lane == 0) {
-        const int64_t g = g0 + u * n_hw;
+        const int64_t t = g0 + u * n_hw;
+        const int64_t g = REVERSE ? g_end - 1 - (t - g_begin) : t;
         const int64_t s = g / a.budget;
         const int64_t j = g - s * a.budget;
         a.pid_dst[s * a.cap + j] = a.pid_src ? a.pid_src[s * a.cap + src_n[u]]

@@ -10,6 +10,14 @@ __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a)
   extern __shared__ uint32_t sm_sel[];
   __shared__ dev::SelShared sh;
   pdl_trigger();
+  // The selection is latency-bound: meanwhile, start moving this slab's
+  // recent rows (always kept) into L2 for the compaction that follows.
+  if (a.k_pf && threadIdx.x < 2) {
+    const int64_t n_past = a.n_tokens - a.rp;
+    const char* base = static_cast<const char*>(threadIdx.x ? a.v_pf : a.k_pf);
+    prefetch_l2(base + (blockIdx.x * a.cap_pf + n_past) * a.row_bytes_pf,
+                static_cast<uint32_t>(a.rp * a.row_bytes_pf));
+  }
   pdl_wait();  // the scores come from the scoring kernel
   dev::select_slab<kSelectThreads>(a, blockIdx.x, sm_sel, sh);
 }
