@@ -9,7 +9,14 @@ Qwen2-VL-7B on long-video benchmarks, which are not available here):
     N(0,1) innovations and a stationary start k_0 ~ N(0, I/(1 - rho^2));
     exactly floor(static_frac * p) patches (a seeded permutation, shared by
     all slabs of a stream) are static (rho_static), the rest dynamic;
-  * values: unit Gaussian directions times LogNormal(0, sigma) magnitudes;
+  * values: unit Gaussian directions times magnitudes exp(sigma_l g), with
+    g = beta_l S + sqrt(1 - beta_l^2) z, z ~ N(0,1) per token and S a smooth
+    unit-variance field over each frame's grid (four random low-frequency
+    cosines per (slab, frame)); sigma_l runs linearly from value_sigma (first
+    layer) to value_sigma_last (last layer) and beta_l from value_locality
+    down to 0, so early layers have tight, spatially clustered value norms
+    and deep layers dispersed, unclustered ones; with the defaults every
+    layer has sigma_l = value_sigma and beta_l = 0 (LogNormal(0, sigma));
   * storage: bf16 (round to nearest even) or fp32, layout [slab][cap][D].
 Random numbers come from Philox4x32-10 (Salmon et al., SC 2011) with
 counter (frame*p + patch, slab, purpose, dim/4) and key (seed, stream), so
@@ -52,6 +59,10 @@ class Workload:
     recent_frames: int = 0  # 0: library default
     stream_frames: int = 0  # streaming run: total frames in the stream
     append_frames: int = 0  # streaming run: frames appended per step
+    value_sigma_last: float | None = None  # sigma of the last layer (None: value_sigma)
+    value_locality: float = 0.0            # beta of the first layer (falls to 0 at the last)
+    van_pool: bool = False                 # layer-adaptive VaN pooling in the pass
+    cv_tau: tuple = (0.0, 0.0, 0.0)        # CV thresholds of the pool-size map
 
     @property
     def p(self) -> int:
@@ -94,7 +105,44 @@ CONFIGS = {
                        stream_frames=3600, append_frames=16),
     # 8 independent streams of an 80-layer x 8-KV-head model, 128 frames of 16x16
     "large": Workload("large", 80, 8, 128, "bf16", 16, 16, 128, 24576, 0.5, n_streams=8),
+    # the LLaVA shape with layer-adaptive VaN pooling: value spread grows and
+    # spatial clustering fades with depth; the CV thresholds split the 28
+    # layers over pool sizes 7, 5, 3 and 1
+    "llava_pool": Workload("llava_pool", 28, 4, 128, "bf16", 14, 14, 48, 6272, 0.5,
+                           value_sigma=0.25, value_sigma_last=1.0, value_locality=0.9,
+                           van_pool=True, cv_tau=(0.4, 0.6, 0.9)),
 }
+
+
+def value_params(w: Workload):
+    """Per-layer (sigma_l, beta_l) as float32 arrays [n_layers], or None when
+    every layer uses value_sigma with no spatial field."""
+    if w.value_sigma_last is None and w.value_locality == 0.0:
+        return None
+    L = w.n_layers
+    frac = np.arange(L, dtype=np.float64) / max(L - 1, 1)
+    last = w.value_sigma if w.value_sigma_last is None else w.value_sigma_last
+    sigma = w.value_sigma + (last - w.value_sigma) * frac
+    beta = w.value_locality * (1.0 - frac) if L > 1 else np.full(1, w.value_locality)
+    return sigma.astype(np.float32), beta.astype(np.float32)
+
+
+def _frame_field(t: int, s_idx, key, gh: int, gw: int) -> np.ndarray:
+    """Smooth unit-variance field [S, gh*gw] of frame t for every slab in s_idx
+    (the device generator's frame_field, in float64)."""
+    S = s_idx.shape[0]
+    w = philox4x32_10((np.uint64(t), s_idx, np.uint64(3), np.uint64(0)), key)
+    ph = philox4x32_10((np.uint64(t), s_idx, np.uint64(4), np.uint64(0)), key)
+    i = (np.arange(gh * gw) // gw).astype(np.float64)[None, :]
+    j = (np.arange(gh * gw) % gw).astype(np.float64)[None, :]
+    acc = np.zeros((S, gh * gw))
+    for a in range(4):
+        wa = np.asarray(w[a]).reshape(S, 1)
+        u = (wa % np.uint64(3)).astype(np.float64)
+        v = ((wa // np.uint64(3)) % np.uint64(3)).astype(np.float64)
+        phi = _unit_open(np.asarray(ph[a]).reshape(S, 1))
+        acc += np.sqrt(0.5) * np.cos(2.0 * np.pi * (u * i / gh + v * j / gw + phi))
+    return acc
 
 
 def patch_rho(w: Workload, stream: int = 0) -> np.ndarray:
@@ -170,6 +218,11 @@ def host_generate(w: Workload, stream: int = 0, n_frames: int | None = None,
     K = np.zeros((S, cap, D), np.float32)
     V = np.zeros((S, cap, D), np.float32)
     x = np.zeros((S, p, D), np.float64)
+    vp = value_params(w)
+    vparams = None
+    if vp is not None:  # per-slab sigma and beta of the slab's layer
+        layer = (np.arange(S) // w.n_kv_heads) % w.n_layers
+        vparams = (vp[0][layer].astype(np.float64), vp[1][layer].astype(np.float64))
     for t in range(f):
         tok = np.uint64(t * p) + q_idx
         z = _four_normals(philox4x32_10((tok, s_idx, np.uint64(0), c_idx), key)).reshape(S, p, D)
@@ -182,7 +235,16 @@ def host_generate(w: Workload, stream: int = 0, n_frames: int | None = None,
         u = _four_normals(philox4x32_10((tok, s_idx, np.uint64(1), c_idx), key)).reshape(S, p, D)
         zm = _four_normals(philox4x32_10((np.uint64(t * p) + q_idx[..., 0], s_idx[..., 0],
                                           np.uint64(2), np.uint64(0)), key))[..., 0]
-        mag = np.exp(w.value_sigma * zm) / np.linalg.norm(u, axis=-1)
+        if vparams is None:
+            mag = np.exp(w.value_sigma * zm) / np.linalg.norm(u, axis=-1)
+        else:
+            sig_s, beta_s = vparams
+            g = zm
+            if np.any(beta_s != 0):
+                field = _frame_field(t, s_idx[:, 0, 0], key, w.grid_h, w.grid_w)
+                g = np.where(beta_s[:, None] != 0,
+                             beta_s[:, None] * field + np.sqrt(1.0 - beta_s[:, None] ** 2) * zm, zm)
+            mag = np.exp(sig_s[:, None] * g) / np.linalg.norm(u, axis=-1)
         V[:, t * p:(t + 1) * p] = u * mag[..., None]
     if w.is_bf16:
         return to_bf16_bits(K), to_bf16_bits(V)
@@ -209,7 +271,8 @@ def _load():
         lib = ctypes.CDLL(_LIB)
         P, I64, I32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
         lib.synth_fill.argtypes = [P, P, I32, I64, I64, I32, I32, I32, I32, I64, P, P,
-                                   ctypes.c_float, ctypes.c_uint64, ctypes.c_uint32, I64, P]
+                                   ctypes.c_float, ctypes.c_uint64, ctypes.c_uint32, I64,
+                                   P, P, I32, I32, I32, P]
         lib.synth_fill.restype = I32
         _lib = lib
     return _lib
@@ -225,6 +288,11 @@ class DeviceGenerator:
         dev = torch.device("cuda") if device is None else device
         self.rho = torch.from_numpy(patch_rho(w, stream)).to(dev)
         self.state = torch.zeros((n_slabs, w.p, w.head_dim), dtype=torch.float32, device=dev)
+        vp = value_params(w)
+        self.layer_sigma = self.layer_beta = None
+        if vp is not None:
+            self.layer_sigma = torch.from_numpy(vp[0]).to(dev)
+            self.layer_beta = torch.from_numpy(vp[1]).to(dev)
         self.next_frame = 0
 
     def fill(self, k, v, row0: int, n_frames: int, slab_base: int = 0):
@@ -235,6 +303,9 @@ class DeviceGenerator:
                                 self.w.p, self.next_frame, n_frames, row0,
                                 self.rho.data_ptr(), self.state.data_ptr(),
                                 self.w.value_sigma, self.w.seed, self.stream, slab_base,
+                                None if self.layer_sigma is None else self.layer_sigma.data_ptr(),
+                                None if self.layer_beta is None else self.layer_beta.data_ptr(),
+                                self.w.n_layers, self.w.n_kv_heads, self.w.grid_w,
                                 torch.cuda.current_stream().cuda_stream)
         if rc != 0:
             raise RuntimeError(f"synth_fill failed with code {rc}")

@@ -6,7 +6,11 @@
 //   keys   per (slab, patch, dim): AR(1) across frames,
 //          k_0 = e_0 / sqrt(1 - rho^2),  k_t = rho k_{t-1} + e_t,  e ~ N(0,1),
 //          rho = rho[patch] (static or dynamic patch, chosen on the host);
-//   values per token: v = (u / ||u||) * exp(sigma z),  u ~ N(0, I_D), z ~ N(0,1);
+//   values per token: v = (u / ||u||) * exp(sigma_l g),  u ~ N(0, I_D), where
+//          g = beta_l S(t,i,j) + sqrt(1 - beta_l^2) z,  z ~ N(0,1), and S is a
+//          smooth unit-variance field over each frame's grid (a sum of four
+//          random low-frequency cosines drawn per (slab, frame)); sigma_l and
+//          beta_l are per-layer (NULL arrays: sigma_l = sigma, beta_l = 0, g = z);
 //   stored as bf16 (round to nearest even) or fp32.
 // Random numbers: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random
 // numbers: as easy as 1, 2, 3", SC 2011), counter = (frame*p + patch, slab,
@@ -101,10 +105,37 @@ __global__ void keys_kernel(T* k, int64_t n_slabs, int64_t cap, int D, int p, in
 }
 
 // One warp per token row: u ~ N(0, I_D) normalised, scaled by a lognormal.
+// Smooth unit-variance field over a frame's gh x gw grid at patch (i, j):
+// sum over a < 4 of sqrt(1/2) cos(2 pi (u_a i / gh + v_a j / gw + phi_a)), with
+// u_a, v_a in {0, 1, 2} and phi_a uniform, drawn once per (slab, frame).
+__device__ float frame_field(uint32_t frame, uint32_t slab, int i, int j, int gh, int gw,
+                             uint32_t key0, uint32_t key1) {
+  const U4 w = philox4x32_10(U4{frame, slab, 3u, 0u}, key0, key1);
+  const U4 ph = philox4x32_10(U4{frame, slab, 4u, 0u}, key0, key1);
+  const uint32_t ws[4] = {w.a, w.b, w.c, w.d};
+  const uint32_t phs[4] = {ph.a, ph.b, ph.c, ph.d};
+  float acc = 0.0f;
+#pragma unroll
+  for (int a = 0; a < 4; ++a) {
+    const float u = static_cast<float>(ws[a] % 3u);
+    const float vv = static_cast<float>((ws[a] / 3u) % 3u);
+    const float x = u * static_cast<float>(i) / static_cast<float>(gh) +
+                    vv * static_cast<float>(j) / static_cast<float>(gw) + unit_open(phs[a]);
+    acc += 0.70710678f * cospif(2.0f * x);
+  }
+  return acc;
+}
+
+struct ValueParams {
+  const float* layer_sigma;  // [n_layers] or NULL
+  const float* layer_beta;   // [n_layers] or NULL
+  int n_layers, n_kv_heads, grid_w;
+};
+
 template <typename T>
 __global__ void values_kernel(T* v, int64_t n_slabs, int64_t cap, int D, int p, int frame0,
                               int n_frames, int64_t row0, float sigma, uint32_t key0,
-                              uint32_t key1, int64_t slab_base) {
+                              uint32_t key1, int64_t slab_base, ValueParams vp) {
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
   const int64_t rows = static_cast<int64_t>(n_frames) * p;
@@ -127,7 +158,20 @@ __global__ void values_kernel(T* v, int64_t n_slabs, int64_t cap, int D, int p, 
   for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
   float zm[4];
   four_normals(philox4x32_10(U4{token, slab, 2u, 0u}, key0, key1), zm);
-  const float scale = expf(sigma * zm[0]) / sqrtf(ss);
+  float sig = sigma, g = zm[0];
+  if (vp.layer_sigma) {
+    const int layer = static_cast<int>((slab / static_cast<uint32_t>(vp.n_kv_heads)) %
+                                       static_cast<uint32_t>(vp.n_layers));
+    sig = vp.layer_sigma[layer];
+    const float beta = vp.layer_beta[layer];
+    if (beta != 0.0f) {
+      const int q = static_cast<int>(token % static_cast<uint32_t>(p));
+      const float field = frame_field(token / static_cast<uint32_t>(p), slab, q / vp.grid_w,
+                                      q % vp.grid_w, p / vp.grid_w, vp.grid_w, key0, key1);
+      g = beta * field + sqrtf(1.0f - beta * beta) * zm[0];
+    }
+  }
+  const float scale = expf(sig * g) / sqrtf(ss);
   T* row = v + (s * cap + row0 + i) * D;
   for (int j = 0; j < 16; ++j) {
     const int c = lane + 32 * j;
@@ -141,7 +185,8 @@ __global__ void values_kernel(T* v, int64_t n_slabs, int64_t cap, int D, int p, 
 template <typename T>
 cudaError_t launch(void* k, void* v, int64_t n_slabs, int64_t cap, int D, int p, int frame0,
                    int n_frames, int64_t row0, const float* rho, float* state, float sigma,
-                   uint64_t seed, uint32_t stream_id, int64_t slab_base, cudaStream_t st) {
+                   uint64_t seed, uint32_t stream_id, int64_t slab_base, ValueParams vp,
+                   cudaStream_t st) {
   const uint32_t key0 = static_cast<uint32_t>(seed);
   const uint32_t key1 = static_cast<uint32_t>(seed >> 32) + stream_id;
   const int64_t kthreads = n_slabs * p * (D / 4);
@@ -151,7 +196,7 @@ cudaError_t launch(void* k, void* v, int64_t n_slabs, int64_t cap, int D, int p,
   const int64_t vwarps = n_slabs * n_frames * static_cast<int64_t>(p);
   values_kernel<T><<<static_cast<unsigned>((vwarps * 32 + 255) / 256), 256, 0, st>>>(
       static_cast<T*>(v), n_slabs, cap, D, p, frame0, n_frames, row0, sigma, key0, key1,
-      slab_base);
+      slab_base, vp);
   return cudaGetLastError();
 }
 
@@ -163,21 +208,29 @@ extern "C" {
 // row0 + (t - frame0) * p + patch of k and v ([n_slabs][cap][D], bf16 or
 // fp32). rho: device [p]. state: device fp32 [n_slabs][p][D] holding the last
 // key of each AR(1) chain (read unless frame0 == 0, always written back).
+// layer_sigma, layer_beta: device fp32 [n_layers] per-layer value spread and
+// spatial weight (both NULL: sigma for every layer, no spatial field); slab
+// s + slab_base belongs to layer ((s + slab_base) / n_kv_heads) mod n_layers.
 // Returns 0 or a cudaError_t value; 1000 for bad arguments.
 int synth_fill(void* k, void* v, int is_bf16, int64_t n_slabs, int64_t cap, int D, int p,
                int frame0, int n_frames, int64_t row0, const float* rho, float* state,
                float sigma, uint64_t seed, uint32_t stream_id, int64_t slab_base,
-               void* stream) {
+               const float* layer_sigma, const float* layer_beta, int n_layers, int n_kv_heads,
+               int grid_w, void* stream) {
   if (!k || !v || !rho || !state || n_slabs <= 0 || D <= 0 || D % 4 != 0 || D > 2048 ||
       p <= 0 || frame0 < 0 || n_frames <= 0 || row0 < 0 ||
       row0 + static_cast<int64_t>(n_frames) * p > cap)
     return 1000;
+  if ((layer_sigma == nullptr) != (layer_beta == nullptr)) return 1000;
+  if (layer_sigma && (n_layers <= 0 || n_kv_heads <= 0 || grid_w <= 0 || p % grid_w != 0))
+    return 1000;
+  const ValueParams vp{layer_sigma, layer_beta, n_layers, n_kv_heads, grid_w};
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (is_bf16)
     return launch<__nv_bfloat16>(k, v, n_slabs, cap, D, p, frame0, n_frames, row0, rho, state,
-                                 sigma, seed, stream_id, slab_base, st);
+                                 sigma, seed, stream_id, slab_base, vp, st);
   return launch<float>(k, v, n_slabs, cap, D, p, frame0, n_frames, row0, rho, state, sigma,
-                       seed, stream_id, slab_base, st);
+                       seed, stream_id, slab_base, vp, st);
 }
 
 }  // extern "C"

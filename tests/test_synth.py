@@ -48,3 +48,26 @@ def test_bf16_rounding_is_nearest_even():
     back = synth.bf16_bits_to_f32(b)
     assert b[1] == 0x3F80 and b[2] == 0x3F82       # ties to even
     assert np.all(np.abs(back - x) <= np.abs(x) * 2 ** -8)
+
+
+def test_layer_varying_values():
+    """Per-layer value spread and spatial clustering (the pooled workload):
+    the log-norm spread of layer l is sigma_l; the smooth field makes
+    neighbouring patches of a frame correlated in early layers only."""
+    w = synth.CONFIGS["llava_pool"].scaled(n_layers=4, n_kv_heads=2, n_frames=16, head_dim=32,
+                                           budget=1000)
+    sig, beta = synth.value_params(w)
+    assert np.allclose(sig, [0.25, 0.5, 0.75, 1.0]) and np.allclose(beta, [0.9, 0.6, 0.3, 0.0])
+    _, V = synth.host_generate(w)
+    V = synth.bf16_bits_to_f32(V).astype(np.float64)
+    ln = np.log(np.linalg.norm(V, axis=-1)).reshape(w.n_layers, w.n_kv_heads, w.n_frames,
+                                                    w.grid_h, w.grid_w)
+    corr = []
+    for layer in range(w.n_layers):
+        x = ln[layer]
+        assert abs(x.std() - sig[layer]) < 0.08 * sig[layer] + 0.02
+        a, b = x[..., :, :-1].ravel(), x[..., :, 1:].ravel()     # horizontal neighbours
+        corr.append(np.corrcoef(a, b)[0, 1])
+    assert corr[0] > 0.5 and abs(corr[-1]) < 0.1 and corr[0] > corr[1] > corr[2]
+    # defaults leave every layer at value_sigma with no field
+    assert synth.value_params(synth.CONFIGS["llava"]) is None
