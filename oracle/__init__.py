@@ -10,6 +10,9 @@ Functions mirror the paper's steps:
   select()  -- split-budget selection (Algorithm 1 steps 3-5, Sec. 3.3)
   gather()  -- compaction K~ = K[:, J, :] (Sec. 3.1, Algorithm 2 last step)
   compress()-- the three in sequence (used to time the oracle)
+  van_all(), pool_size(), van_pool(), compress_pooled()
+            -- layer-adaptive VaN pooling (Sec. 3.2, Algorithm 2) and the pass
+               whose VaN stage ranks pooled VaN
 """
 from __future__ import annotations
 
@@ -61,8 +64,16 @@ def _load():
         lib.oracle_gather_patch.argtypes = [P, P, I64, I64, I64, I32, P, I64]
         lib.oracle_gather_patch.restype = I32
         lib.oracle_compress.argtypes = [P, P, I32, I64, I64, I32, I64, I32, I32, I64, D,
-                                        P, P, P, P, P]
+                                        P, P, P, P, P, I32, P, I32, I32, P, P, P]
         lib.oracle_compress.restype = I32
+        lib.oracle_gather_frame.argtypes = [P, P, I64, I64, I64, I32, P, I64]
+        lib.oracle_gather_frame.restype = I32
+        lib.oracle_van_all.argtypes = [P, I32, I64, I64, I32, I64, P]
+        lib.oracle_van_all.restype = I32
+        lib.oracle_pool_size.argtypes = [D, P]
+        lib.oracle_pool_size.restype = I32
+        lib.oracle_van_pool.argtypes = [P, I64, I32, I64, I32, I32, P, P, I64, P, P, P, P]
+        lib.oracle_van_pool.restype = I32
         _lib = lib
     return _lib
 
@@ -175,7 +186,78 @@ def compress(k: np.ndarray, v: np.ndarray, n_tokens: int, p: int, r: int, budget
         patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
     rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
                                  budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
-                                 _ptr(pd), _ptr(kept))
+                                 _ptr(pd), _ptr(kept), 0, None, 1, 0, None, None, None)
     if rc != 0:
         raise ValueError("oracle_compress rejected its arguments")
     return kept, kd, vd, pd
+
+
+def _tau(tau) -> np.ndarray:
+    t = np.ascontiguousarray(tau, dtype=np.float64)
+    assert t.shape == (3,)
+    return t
+
+
+def van_all(v: np.ndarray, n_tokens: int) -> np.ndarray:
+    """VaN of every row 0..n_tokens-1 (recent frames included), fp64 [S, n_tokens]."""
+    v = np.ascontiguousarray(v)
+    S, cap, D = v.shape
+    out = np.empty((S, n_tokens), np.float64)
+    if _load().oracle_van_all(_ptr(v), _kv_kind(v), S, cap, D, n_tokens, _ptr(out)) != 0:
+        raise ValueError("oracle_van_all rejected its arguments")
+    return out
+
+
+def pool_size(cv: float, tau) -> int:
+    """g(CV) of Algorithm 2 for thresholds tau = (tau_1, tau_2, tau_3)."""
+    return _load().oracle_pool_size(float(cv), _ptr(_tau(tau)))
+
+
+def van_pool(van: np.ndarray, n_kv_heads: int, grid_h: int, grid_w: int, tau,
+             patch_id: np.ndarray | None = None, frame_id: np.ndarray | None = None):
+    """Layer-adaptive pooled VaN (Sec. 3.2, Algorithm 2) of van [S, N] (every
+    cached row). Returns (pooled [S, N], pool size per layer, CV per layer)."""
+    van = np.ascontiguousarray(van, dtype=np.float64)
+    S, N = van.shape
+    stride = N
+    if patch_id is not None:
+        patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
+        frame_id = np.ascontiguousarray(frame_id, dtype=np.uint32)
+        assert patch_id.shape == frame_id.shape and patch_id.shape[0] == S
+        stride = patch_id.shape[1]
+    pooled = np.empty_like(van)
+    L = S // n_kv_heads
+    ks = np.empty(L, np.int32)
+    cvs = np.empty(L, np.float64)
+    rc = _load().oracle_van_pool(_ptr(van), S, n_kv_heads, N, grid_h, grid_w, _ptr(patch_id),
+                                 _ptr(frame_id), stride, _ptr(_tau(tau)), _ptr(pooled),
+                                 _ptr(ks), _ptr(cvs))
+    if rc != 0:
+        raise ValueError("oracle_van_pool rejected its arguments")
+    return pooled, ks, cvs
+
+
+def compress_pooled(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, grid_w: int,
+                    r: int, budget: int, alpha: float, tau, n_kv_heads: int,
+                    patch_id: np.ndarray | None = None, frame_id: np.ndarray | None = None):
+    """Whole pass whose VaN stage ranks layer-adaptive pooled VaN. Returns
+    (kept, K~, V~, patch ids, frame ids, pool size per layer)."""
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    S, cap, D = k.shape
+    p = grid_h * grid_w
+    kd, vd = np.zeros_like(k), np.zeros_like(v)
+    pd = np.zeros((S, cap), np.uint16)
+    fd = np.zeros((S, cap), np.uint32)
+    kept = np.empty((S, budget), np.int32)
+    ks = np.zeros(S // n_kv_heads, np.int32)
+    if patch_id is not None:
+        patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
+        frame_id = np.ascontiguousarray(frame_id, dtype=np.uint32)
+    rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
+                                 budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
+                                 _ptr(pd), _ptr(kept), 1, _ptr(_tau(tau)), n_kv_heads,
+                                 grid_w, _ptr(frame_id), _ptr(fd), _ptr(ks))
+    if rc != 0:
+        raise ValueError("oracle_compress rejected its arguments")
+    return kept, kd, vd, pd, fd, ks

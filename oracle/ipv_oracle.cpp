@@ -32,6 +32,18 @@
 // past-token patch coordinates come from an optional per-token patch-id array
 // (else n mod p), recent rows are whole frames at rows N - r p + t' p + q.
 //
+// Layer-adaptive VaN pooling (Sec. 3.2 "Layer-wise Adaptive Pooling";
+// Algorithm 2), used when the pass is asked for it: per layer, the mean mu and
+// standard deviation sigma of VaN over all heads and all cached tokens give
+// CV = sigma / mu; g(CV) = 7, 5, 3, 1 for CV < tau_1, < tau_2, < tau_3, >= tau_3
+// picks an average-pool size k; each token's pooled VaN is the mean VaN of the
+// tokens of its own frame inside the k x k window centred on its grid position
+// (stride 1). Readings: sigma is the population standard deviation; window
+// positions outside the grid, or whose token is no longer cached, are left
+// out of the mean (no zero padding); the VaN stage of the selection ranks the
+// pooled values. Where rows carry patch ids they also carry frame ids (the
+// frame each token came from); a never-compacted cache has frame n div p.
+//
 // Element types: bf16 (widened exactly: bits << 16) or fp32, widened to double.
 
 #include <algorithm>
@@ -39,6 +51,7 @@
 #include <cstdint>
 #include <cstring>
 #include <limits>
+#include <map>
 #include <vector>
 
 namespace {
@@ -258,18 +271,148 @@ int oracle_gather_patch(const uint16_t* src_pid, uint16_t* dst_pid, int64_t n_sl
   return 0;
 }
 
+// Frame ids travel with their tokens: dst[s][j] = src ? src[s][kept] : kept div p.
+int oracle_gather_frame(const uint32_t* src_fid, uint32_t* dst_fid, int64_t n_slabs,
+                        int64_t cap_src, int64_t cap_dst, int p,
+                        const int32_t* kept, int64_t budget) {
+  if (!dst_fid || !kept || p <= 0) return -1;
+  for (int64_t s = 0; s < n_slabs; ++s)
+    for (int64_t j = 0; j < budget; ++j) {
+      const int32_t n = kept[s * budget + j];
+      if (n < 0) continue;
+      dst_fid[s * cap_dst + j] =
+          src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n / p);
+    }
+  return 0;
+}
+
+// VaN of every cached row, recent frames included (Algorithm 2 takes mu and
+// sigma over the whole layer's ||V_l||_2). van_out: [n_slabs][n_tokens].
+int oracle_van_all(const void* v, int is_bf16, int64_t n_slabs, int64_t cap, int D,
+                   int64_t n_tokens, double* van_out) {
+  if (!v || !van_out || n_slabs < 0 || D <= 0 || n_tokens < 0 || n_tokens > cap) return -1;
+  std::vector<double> vv;
+  for (int64_t s = 0; s < n_slabs; ++s)
+    for (int64_t n = 0; n < n_tokens; ++n) {
+      load_row(v, is_bf16, s, cap, D, n, vv);
+      van_out[s * n_tokens + n] = l2norm(vv);
+    }
+  return 0;
+}
+
+// Pool size g(CV) of Algorithm 2: 7 if CV < tau_1, 5 if tau_1 <= CV < tau_2,
+// 3 if tau_2 <= CV < tau_3, 1 if CV >= tau_3. A NaN CV satisfies none of the
+// strict comparisons and gets 1 (no pooling).
+int oracle_pool_size(double cv, const double* tau) {
+  if (cv < tau[0]) return 7;
+  if (cv < tau[1]) return 5;
+  if (cv < tau[2]) return 3;
+  return 1;
+}
+
+// Layer-adaptive pooling of VaN (Sec. 3.2; Algorithm 2). van: [n_slabs][n_tokens]
+// VaN of every cached row; slabs s = l * n_kv_heads + h form layer l.
+// patch_id (uint16) and frame_id (uint32), both [n_slabs][id_stride] or both
+// NULL (then row n is patch n mod p of frame n div p). For each layer:
+//   mu = mean, sigma = population std of all its heads' VaN values,
+//   CV = sigma / mu, k = g(CV);
+// for each row n of each of its slabs, at frame F and grid position (i, j)
+// (patch q = i * grid_w + j):
+//   k == 1: pooled = VaN[n];
+//   k  > 1: pooled = mean of VaN[m] over the rows m of the same slab and
+//           frame F whose position (i', j') has |i' - i| <= k div 2 and
+//           |j' - j| <= k div 2 (row n itself included);
+//   a patch id >= p has no position: its pooled value is NaN (k > 1).
+// pooled_out: [n_slabs][n_tokens]; pool_size_out, cv_out: [n_layers] or NULL.
+int oracle_van_pool(const double* van, int64_t n_slabs, int n_kv_heads, int64_t n_tokens,
+                    int grid_h, int grid_w, const uint16_t* patch_id,
+                    const uint32_t* frame_id, int64_t id_stride, const double* tau,
+                    double* pooled_out, int32_t* pool_size_out, double* cv_out) {
+  if (!van || !pooled_out || !tau || n_kv_heads <= 0 || n_slabs % n_kv_heads != 0 ||
+      n_tokens <= 0 || grid_h <= 0 || grid_w <= 0 || (patch_id == nullptr) != (frame_id == nullptr) ||
+      (patch_id && id_stride < n_tokens))
+    return -1;
+  const int64_t p = static_cast<int64_t>(grid_h) * grid_w;
+  const double nan = std::numeric_limits<double>::quiet_NaN();
+  const int64_t n_layers = n_slabs / n_kv_heads;
+  for (int64_t l = 0; l < n_layers; ++l) {
+    const double* lv = van + l * n_kv_heads * n_tokens;
+    const int64_t count = n_kv_heads * n_tokens;
+    double sum = 0.0;
+    for (int64_t i = 0; i < count; ++i) sum += lv[i];
+    const double mu = sum / static_cast<double>(count);
+    double ss = 0.0;
+    for (int64_t i = 0; i < count; ++i) ss += (lv[i] - mu) * (lv[i] - mu);
+    const double sigma = std::sqrt(ss / static_cast<double>(count));
+    const double cv = sigma / mu;
+    const int k = oracle_pool_size(cv, tau);
+    if (pool_size_out) pool_size_out[l] = k;
+    if (cv_out) cv_out[l] = cv;
+    const int64_t half = k / 2;
+    for (int64_t h = 0; h < n_kv_heads; ++h) {
+      const int64_t s = l * n_kv_heads + h;
+      const double* sv = van + s * n_tokens;
+      double* out = pooled_out + s * n_tokens;
+      if (k == 1) {
+        for (int64_t n = 0; n < n_tokens; ++n) out[n] = sv[n];
+        continue;
+      }
+      std::vector<int64_t> frame(n_tokens), patch(n_tokens);
+      std::map<int64_t, std::vector<int64_t>> rows_of_frame;
+      for (int64_t n = 0; n < n_tokens; ++n) {
+        frame[n] = patch_id ? static_cast<int64_t>(frame_id[s * id_stride + n]) : n / p;
+        patch[n] = patch_id ? static_cast<int64_t>(patch_id[s * id_stride + n]) : n % p;
+        rows_of_frame[frame[n]].push_back(n);
+      }
+      for (int64_t n = 0; n < n_tokens; ++n) {
+        if (patch[n] >= p) {
+          out[n] = nan;
+          continue;
+        }
+        const int64_t i = patch[n] / grid_w, j = patch[n] % grid_w;
+        double acc = 0.0;
+        int64_t cnt = 0;
+        for (int64_t m : rows_of_frame[frame[n]]) {
+          if (patch[m] >= p) continue;
+          const int64_t im = patch[m] / grid_w, jm = patch[m] % grid_w;
+          if (std::llabs(im - i) <= half && std::llabs(jm - j) <= half) {
+            acc += sv[m];
+            ++cnt;
+          }
+        }
+        out[n] = acc / static_cast<double>(cnt);
+      }
+    }
+  }
+  return 0;
+}
+
 // One whole pass over slabs [0, n_slabs): scores, selection, compaction of K
-// and V (and of patch ids when dst_pid != NULL). Used to time the oracle.
+// and V (and of patch ids when dst_pid != NULL, of frame ids when dst_fid !=
+// NULL). With van_pool != 0 the VaN stage ranks the layer-adaptive pooled
+// VaN (tau: the three CV thresholds; n_kv_heads groups slabs into layers;
+// src_fid goes with src_pid). pool_size_out: [n_slabs / n_kv_heads] or NULL.
 int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
                     int64_t cap, int D, int64_t n_tokens, int p, int r,
                     int64_t budget, double alpha, const uint16_t* src_pid,
-                    void* k_dst, void* v_dst, uint16_t* dst_pid, int32_t* kept_out) {
+                    void* k_dst, void* v_dst, uint16_t* dst_pid, int32_t* kept_out,
+                    int van_pool, const double* tau, int n_kv_heads, int grid_w,
+                    const uint32_t* src_fid, uint32_t* dst_fid, int32_t* pool_size_out) {
   std::vector<double> tar(static_cast<size_t>(n_slabs * n_tokens));
   std::vector<double> van(tar.size());
   if (n_tokens > budget) {
     if (oracle_scores(k, v, is_bf16, n_slabs, cap, D, n_tokens, p, r, src_pid,
                       tar.data(), van.data()) != 0)
       return -1;
+    if (van_pool) {
+      if (grid_w <= 0 || p % grid_w != 0) return -1;
+      std::vector<double> all(tar.size());
+      if (oracle_van_all(v, is_bf16, n_slabs, cap, D, n_tokens, all.data()) != 0) return -1;
+      if (oracle_van_pool(all.data(), n_slabs, n_kv_heads, n_tokens, p / grid_w, grid_w,
+                          src_pid, src_fid, cap, tau, van.data(), pool_size_out,
+                          nullptr) != 0)
+        return -1;
+    }
   }
   if (oracle_select(tar.data(), van.data(), n_slabs, n_tokens, p, r, budget, alpha,
                     kept_out, nullptr) != 0)
@@ -280,6 +423,9 @@ int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
   if (oracle_gather_rows(v, v_dst, row_bytes, n_slabs, cap, cap, kept_out, budget) != 0) return -1;
   if (dst_pid &&
       oracle_gather_patch(src_pid, dst_pid, n_slabs, cap, cap, p, kept_out, budget) != 0)
+    return -1;
+  if (dst_fid &&
+      oracle_gather_frame(src_fid, dst_fid, n_slabs, cap, cap, p, kept_out, budget) != 0)
     return -1;
   return 0;
 }

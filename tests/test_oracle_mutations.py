@@ -2,7 +2,8 @@
 
 Each case plants one mistake (a flipped sign, a dropped term, a wrong index,
 a wrong tie-break, ...) in a copy of oracle/ipv_oracle.cpp, builds the copy on
-the CPU, and runs the pin suite (test_oracle_pins.py) against it. Every
+the CPU, and runs the pin suites (test_oracle_pins.py, test_oracle_pool_pins.py)
+against it. Every
 mutant must make that suite fail; the unmutated copy must pass it.
 """
 import os
@@ -26,8 +27,10 @@ MUTANTS = [
     ("cosine misses the past-key norm",
      "std::max(l2norm(a), eps) * std::max(l2norm(b), eps)", "std::max(l2norm(b), eps)"),
     ("VaN squared norm", "van[n] = l2norm(vv);", "van[n] = dot(vv, vv);"),
-    ("VaN scored on keys", "load_row(v, is_bf16, s, cap, D, n, vv);",
-     "load_row(k, is_bf16, s, cap, D, n, vv);"),
+    ("VaN scored on keys", "load_row(v, is_bf16, s, cap, D, n, vv);\n      van[n] =",
+     "load_row(k, is_bf16, s, cap, D, n, vv);\n      van[n] ="),
+    ("all-row VaN squared", "van_out[s * n_tokens + n] = l2norm(vv);",
+     "van_out[s * n_tokens + n] = dot(vv, vv);"),
     ("ties go to the higher index", "  return xi < yi;\n}\n\n}  // namespace",
      "  return xi > yi;\n}\n\n}  // namespace"),
     ("lower score wins", "if (xs != ys) return xs > ys;", "if (xs != ys) return xs < ys;"),
@@ -41,13 +44,38 @@ MUTANTS = [
     ("default r not rounded", "n_frames / 8.0 + 0.5", "n_frames / 8.0"),
     ("recent tokens not kept", "for (int64_t n = n_past; n < n_tokens; ++n) keep[n] = 1;",
      "for (int64_t n = n_past; n + 1 < n_tokens; ++n) keep[n] = 1;"),
+    # layer-adaptive VaN pooling
+    ("pool mean counts padded positions", "out[n] = acc / static_cast<double>(cnt);",
+     "out[n] = acc / static_cast<double>(k * k);"),
+    ("pool window one cell too wide", "const int64_t half = k / 2;",
+     "const int64_t half = (k + 1) / 2;"),
+    ("pool grid rows and columns swapped",
+     "const int64_t i = patch[n] / grid_w, j = patch[n] % grid_w;",
+     "const int64_t i = patch[n] % grid_h, j = patch[n] / grid_h;"),
+    ("CV with the sample standard deviation", "std::sqrt(ss / static_cast<double>(count))",
+     "std::sqrt(ss / static_cast<double>(count - 1))"),
+    ("CV of one head instead of the layer", "const int64_t count = n_kv_heads * n_tokens;",
+     "const int64_t count = n_tokens;"),
+    ("pool-size threshold inclusive", "if (cv < tau[0]) return 7;", "if (cv <= tau[0]) return 7;"),
+    ("frames of a fresh cache merged", "static_cast<int64_t>(frame_id[s * id_stride + n]) : n / p;",
+     "static_cast<int64_t>(frame_id[s * id_stride + n]) : 0;"),
+    ("frame ids ignored", "frame[n] = patch_id ? static_cast<int64_t>(frame_id[s * id_stride + n])",
+     "frame[n] = patch_id ? static_cast<int64_t>(0)"),
+    ("CV without the recent frames", "if (oracle_van_pool(all.data(),",
+     "if (oracle_van_pool(van.data(),"),
+    ("selection ranks raw VaN", "tau, van.data(), pool_size_out,",
+     "tau, all.data(), pool_size_out,"),
+    ("frame ids of a fresh cache compacted as patch ids",
+     "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n / p)",
+     "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n % p)"),
 ]
 
 
 def _run_pins_with(lib_path: str) -> int:
     env = dict(os.environ, IPV_ORACLE_LIB_OVERRIDE=lib_path)
     cmd = [sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
-           os.path.join(ROOT, "tests", "test_oracle_pins.py")]
+           os.path.join(ROOT, "tests", "test_oracle_pins.py"),
+           os.path.join(ROOT, "tests", "test_oracle_pool_pins.py")]
     return subprocess.run(cmd, env=env, cwd=ROOT, capture_output=True, timeout=300).returncode
 
 
