@@ -27,14 +27,17 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "compress-pass latency (ms) and HBM GB/s vs GB300 peak, 7B shape 6K budget"
-KERNELS = ("recent_mean", "score", "select", "gather", "pipeline")
+KERNELS = ("recent_mean", "score", "select", "gather", "pipeline", "pool")
 FALLBACK_HBM_GBS = 6800.0
 
 
 def workload_desc(w: synth.Workload) -> str:
-    return (f"{w.name}: {w.n_streams}x{w.n_layers} layers x {w.n_kv_heads} KV heads x "
-            f"head_dim {w.head_dim} {w.dtype}, {w.grid_h}x{w.grid_w} tokens/frame, "
-            f"{w.n_frames} frames ({w.n_tokens} tokens) -> budget {w.budget}, alpha {w.tar_ratio}")
+    d = (f"{w.name}: {w.n_streams}x{w.n_layers} layers x {w.n_kv_heads} KV heads x "
+         f"head_dim {w.head_dim} {w.dtype}, {w.grid_h}x{w.grid_w} tokens/frame, "
+         f"{w.n_frames} frames ({w.n_tokens} tokens) -> budget {w.budget}, alpha {w.tar_ratio}")
+    if w.van_pool:
+        d += f", layer-adaptive pooled VaN (CV thresholds {tuple(w.cv_tau)})"
+    return d
 
 
 def peaks():
@@ -60,8 +63,24 @@ def bytes_model(w: synth.Workload, S: int, r: int):
         "select": S * (8 * n_past + 4 * C),
         "gather": S * (4 * C * row + 4 * C),
         "pipeline": pass_bytes,  # the single-kernel pass does all four steps
+        "pool": 0,
     }
+    if w.van_pool:
+        # the recent rows' V (and their VaN) for the layer's CV; the pooling
+        # reads the VaN of every row and writes the pooled VaN of past rows
+        per_kernel["recent_mean"] += S * (rp * row + 4 * rp)
+        per_kernel["pool"] = S * (4 * N + 4 * n_past)
     return pass_bytes, tight, per_kernel
+
+
+def oracle_pass(w: synth.Workload, k_np, v_np, r: int):
+    """One oracle pass over the given slabs (pooled VaN if the workload asks
+    for it; then the slabs are whole layers)."""
+    import oracle
+    if w.van_pool:
+        return oracle.compress_pooled(k_np, v_np, w.n_tokens, w.grid_h, w.grid_w, r, w.budget,
+                                      w.tar_ratio, w.cv_tau, w.n_kv_heads)
+    return oracle.compress(k_np, v_np, w.n_tokens, w.p, r, w.budget, w.tar_ratio)
 
 
 def dram_min_bytes(w: synth.Workload, S: int, r: int) -> int:
@@ -154,12 +173,14 @@ def time_oracle(w: synth.Workload, k_np, v_np, r: int, budget_s: float = 12.0):
     import oracle
     oracle.build()
     S_total = w.n_slabs
+    unit = w.n_kv_heads if w.van_pool else 1  # pooled VaN needs whole layers
     t0 = time.perf_counter()
-    oracle.compress(k_np[:1], v_np[:1], w.n_tokens, w.p, r, w.budget, w.tar_ratio)
-    t1 = time.perf_counter() - t0
+    oracle_pass(w, k_np[:unit], v_np[:unit], r)
+    t1 = (time.perf_counter() - t0) / unit
     n = int(max(1, min(k_np.shape[0], round(budget_s / max(t1, 1e-6)))))
+    n = max(unit, n // unit * unit)
     t0 = time.perf_counter()
-    oracle.compress(k_np[:n], v_np[:n], w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+    oracle_pass(w, k_np[:n], v_np[:n], r)
     dt = time.perf_counter() - t0
     ms_pass = dt * 1e3 * S_total / n
     return ms_pass, n, dt
@@ -173,21 +194,22 @@ def run_reference(args, w: synth.Workload):
     import oracle
     oracle.build()
     r = oracle.recent_frames(w.n_frames)
-    K1, V1 = synth.host_generate(w.scaled(n_layers=1, n_kv_heads=1, n_streams=1))
+    unit = w.n_kv_heads if w.van_pool else 1  # pooled VaN needs whole layers
+    K1, V1 = synth.host_generate(w.scaled(n_streams=1), slabs=unit)
     t0 = time.perf_counter()
-    oracle.compress(K1, V1, w.n_tokens, w.p, r, w.budget, w.tar_ratio)
-    t_slab = time.perf_counter() - t0
+    oracle_pass(w, K1, V1, r)
+    t_slab = (time.perf_counter() - t0) / unit
     # Slabs per step: at most --ref-slabs, fewer if the run would exceed ~2 min.
     fit = int(120.0 / max(1e-6, (args.steps + args.warmup) * t_slab))
     per_step_slabs = max(1, min(w.slabs_per_stream, args.ref_slabs, fit))
-    ws = w.scaled(n_layers=1, n_kv_heads=per_step_slabs, n_streams=1)
-    K, V = synth.host_generate(ws)
+    per_step_slabs = max(unit, per_step_slabs // unit * unit)
+    K, V = synth.host_generate(w.scaled(n_streams=1), slabs=per_step_slabs)
     for _ in range(args.warmup):
-        oracle.compress(K[:1], V[:1], w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+        oracle_pass(w, K[:unit], V[:unit], r)
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        oracle.compress(K, V, w.n_tokens, w.p, r, w.budget, w.tar_ratio)
+        oracle_pass(w, K, V, r)
         times.append(time.perf_counter() - t0)
     ms = float(np.mean(times)) * 1e3 * w.n_slabs / per_step_slabs
     sample = (f"{per_step_slabs} of {w.n_slabs} slabs per step (host-generated, same recipe), "
@@ -261,13 +283,14 @@ def run_stream(args, w: synth.Workload):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     S, N, C, D, p = w.slabs_per_stream, w.n_tokens, w.budget, w.head_dim, w.p
     ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
-             token_capacity=N, single_kernel=args.single_kernel)
+             token_capacity=N, single_kernel=args.single_kernel, van_pool=w.van_pool,
+             cv_tau=w.cv_tau)
     r = ipv.recent_frames(w.n_frames)
     kept = torch.empty((S, C), dtype=torch.int32, device="cuda")
     pid_block = torch.arange(w.append_frames * p, device="cuda").remainder(p).to(torch.int16)
 
     def stream(timed: bool, profile_passes: int = 0):
-        cache = PingPongCache(S, N, D, w.dtype, patch_ids=True)
+        cache = PingPongCache(S, N, D, w.dtype, patch_ids=True, frame_ids=w.van_pool)
         gen = synth.DeviceGenerator(w, S, stream=rank)
         evs, frames, n_pass = [], 0, 0
         t0 = torch.cuda.Event(enable_timing=True)
@@ -278,6 +301,9 @@ def run_stream(args, w: synth.Workload):
             row0 = cache.n_tokens
             gen.fill(cache.k_live, cache.v_live, row0, nf)
             cache.pid_live[:, row0:row0 + nf * p] = pid_block[:nf * p]
+            if cache.fid is not None:  # frame ids: the stream's frame counter
+                cache.fid[cache.cur][:, row0:row0 + nf * p] = (
+                    torch.arange(frames, frames + nf, dtype=torch.int32, device="cuda").repeat_interleave(p))
             cache.n_tokens += nf * p
             frames += nf
             if cache.n_tokens >= N:
@@ -329,9 +355,8 @@ def run_stream(args, w: synth.Workload):
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             n_s = min(S, 16)  # the first pass's input shape, generated on the host
-            K, V = synth.host_generate(w.scaled(n_layers=1, n_kv_heads=n_s))
-            ms_cpu, n_used, secs = time_oracle(w.scaled(n_layers=1, n_kv_heads=S), K, V, r,
-                                               args.cpu_seconds)
+            K, V = synth.host_generate(w, slabs=n_s)
+            ms_cpu, n_used, secs = time_oracle(w, K, V, r, args.cpu_seconds)
             cpu = {"value": ms_cpu, "unit": "ms", "cores": 1, "kind": "oracle",
                    "sample": f"{n_used} of {S} slabs of one pass ({secs:.1f} s, single thread), "
                              f"extrapolated x{S / n_used:.1f} to a full pass",
@@ -400,7 +425,8 @@ def run_gpu(args, w: synth.Workload):
     N, C, D, p = w.n_tokens, w.budget, w.head_dim, w.p
 
     ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
-             token_capacity=N, single_kernel=args.single_kernel)
+             token_capacity=N, single_kernel=args.single_kernel, van_pool=w.van_pool,
+             cv_tau=w.cv_tau)
     r = ipv.recent_frames(w.n_frames)
     cache = PingPongCache(S, N, D, w.dtype, patch_ids=False)
     for i, st in enumerate(streams):

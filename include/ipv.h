@@ -16,6 +16,13 @@
  *         TopK); ties go to the lower token index, NaN ranks lowest;
  *   (iv)  compacts K and V to the kept rows in ascending index order
  *         (Sec. 3.1, K~ = K[:, I, :]; Algorithm 2 last step).
+ * Optionally (ipv_options.van_pool) step (iii) ranks a layer-adaptive average
+ * pooling of VaN instead of raw VaN (Sec. 3.2 "Layer-wise Adaptive Pooling";
+ * Algorithm 2): per layer, CV = sigma/mu of VaN over all its heads and cached
+ * tokens picks a pool size k = g(CV) in {7, 5, 3, 1}, and a token's pooled
+ * VaN is the mean VaN of the cached tokens of its own frame within the k x k
+ * window around its grid position (stride 1; positions outside the grid or
+ * no longer cached are left out; sigma is the population deviation).
  *
  * Memory layout (all device memory, owned by the caller unless stated):
  *   K or V cache half : [n_layers][n_kv_heads][token_capacity][head_dim],
@@ -24,6 +31,9 @@
  *                       element (s * token_capacity + n) * head_dim.
  *   patch ids         : uint16 [n_layers][n_kv_heads][token_capacity]: the
  *                       frame-grid position (i*w + j) of each cached token.
+ *   frame ids         : uint32, same layout: the frame each cached token came
+ *                       from (only equality matters). Pooled VaN needs them
+ *                       once the cache has been compacted.
  *   scores            : fp32 [n_slabs][n_tokens].
  *   kept indices      : int32 [n_slabs][budget], ascending per slab.
  *
@@ -31,7 +41,10 @@
  * tokens (p = frame_grid_h * frame_grid_w). The last r*p rows are the r most
  * recent frames, whole and in patch order. The patch of a past row n is
  * patch_id[n] when the cache half has patch ids, else n mod p (a cache that
- * has never been compacted).
+ * has never been compacted); likewise its frame is frame_id[n], else n div p.
+ * With ids, rows are in increasing (frame id, patch id) order, as appending
+ * whole frames with increasing frame ids and this pass's in-order compaction
+ * keep them (pooled VaN relies on it; no check is made).
  *
  * Execution: every compute entry point validates its arguments on the host,
  * then enqueues kernels on the given CUDA stream and returns without waiting.
@@ -74,18 +87,32 @@ typedef struct {
                              one after the other; 1: as one persistent kernel whose
                              blocks overlap the steps of different slabs. Both give
                              bit-identical results. */
+  int van_pool;           /* 0: the VaN stage ranks raw VaN (Sec. 3.2 s_VaN);
+                             1: it ranks layer-adaptive pooled VaN (Sec. 3.2,
+                             Algorithm 2); needs single_kernel = 0 and
+                             max_frame_tokens <= IPV_MAX_POOL_FRAME_TOKENS */
+  float cv_tau[3];        /* tau_1 <= tau_2 <= tau_3 (van_pool = 1): pool size
+                             g(CV) = 7 if CV < tau_1, 5 if CV < tau_2, 3 if
+                             CV < tau_3, else 1 (Algorithm 2; the paper's values
+                             are model-specific and unpublished) */
 } ipv_options;
 
 /* One tensor (K or V) of the ping-pong cache: two halves of identical
- * layout; buf[cur] holds the live rows. patch_id[h] may be NULL. */
+ * layout; buf[cur] holds the live rows. patch_id[h] and frame_id[h] may be
+ * NULL. */
 typedef struct {
   void* buf[2];
   uint16_t* patch_id[2];
   int cur;
+  uint32_t* frame_id[2];
 } ipv_kv;
 
 /* Largest n_tokens the selection kernel accepts (its keys live in shared memory). */
 #define IPV_MAX_TOKENS 49152
+/* Largest frame (frame_grid_h*frame_grid_w) pooled VaN accepts; the grid
+ * must also satisfy (frame_grid_h + 6) * (frame_grid_w + 6) <= 14080 (a
+ * frame's VaN map, with a 3-cell border, is held in shared memory per warp). */
+#define IPV_MAX_POOL_FRAME_TOKENS 4096
 
 /* Initialise the library on opt->device: checks the device, allocates the
  * scratch (per-token scores and per-patch recent-frame means, sized from
@@ -103,7 +130,9 @@ void ipv_shutdown(void);
  *                   buf[1-cur] and cur is flipped (host-side) in both structs.
  *                   Patch ids: read from k->patch_id[k->cur] (NULL: n mod p);
  *                   written to k->patch_id[1-k->cur] if it is not NULL.
- *                   v->patch_id is not used.
+ *                   Frame ids likewise (k->frame_id; NULL: n div p); with
+ *                   van_pool a cache with patch ids must have frame ids.
+ *                   v->patch_id and v->frame_id are not used.
  *   n_tokens      : |M|, rows currently cached per slab; multiple of p.
  *   budget        : |C|, rows kept per slab; r*p < budget.
  *   tar_ratio     : alpha in [0, 1]; the TaR share is floor(alpha * budget).
@@ -116,7 +145,8 @@ void ipv_shutdown(void);
  * sizes, n_tokens not a multiple of p or above token_capacity or
  * IPV_MAX_TOKENS, budget above token_capacity, tar_ratio outside [0,1] or NaN,
  * r*p >= budget, head_dim*elem_size not a multiple of 16 bytes, sizes above
- * the ipv_init maxima, NULL or misaligned pointers, the two halves aliasing),
+ * the ipv_init maxima, NULL or misaligned pointers, the two halves aliasing,
+ * van_pool with patch ids but no frame ids or a grid too large for pooling),
  * IPV_ENOINIT, IPV_ECUDA (launch failure). */
 ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int head_dim,
                         int64_t n_tokens, int frame_grid_h, int frame_grid_w, int64_t budget,
@@ -124,9 +154,11 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
 
 /* Steps (i) and (ii) only, for inspection and parity checks: fp32 s_TaR and
  * s_VaN of every token of every slab into tar_out / van_out (device,
- * [n_slabs][n_tokens]). Entries of the r recent frames are written as 0.
- * Requires n_tokens > r*p. Same argument rules as ipv_compress (budget and
- * tar_ratio aside); the caches are only read. */
+ * [n_slabs][n_tokens]). Entries of the r recent frames are written as 0,
+ * except that with van_pool van_out holds the VaN of recent rows too (the
+ * layer's CV counts every cached token). Requires n_tokens > r*p. Same
+ * argument rules as ipv_compress (budget and tar_ratio aside); the caches are
+ * only read. */
 ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_heads,
                      int head_dim, int64_t n_tokens, int frame_grid_h, int frame_grid_w,
                      float* tar_out, float* van_out, void* stream);
@@ -137,6 +169,30 @@ ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_he
 ipv_status ipv_select(const float* tar, const float* van, int64_t n_slabs, int64_t n_tokens,
                       int frame_grid_h, int frame_grid_w, int64_t budget, float tar_ratio,
                       int32_t* kept_idx_out, void* stream);
+
+/* The pooling of VaN alone (Sec. 3.2 "Layer-wise Adaptive Pooling";
+ * Algorithm 2 CV, g and AveragePool2d steps), for inspection and parity
+ * checks; the pass runs the same kernel. Works for either van_pool setting.
+ *   van          : device fp32 [n_layers*n_kv_heads][n_tokens]: VaN of every
+ *                  cached row (norms: non-negative or NaN); slabs
+ *                  l*n_kv_heads .. l*n_kv_heads + n_kv_heads-1 form layer l.
+ *   patch_id, frame_id : device [n_slabs][id_stride] uint16 / uint32, both
+ *                  NULL (row n is patch n mod p of frame n div p) or both set,
+ *                  rows in increasing (frame, patch) order.
+ *   cv_tau       : host, the three thresholds (tau_1 <= tau_2 <= tau_3).
+ *   pooled_out   : device fp32 [n_slabs][n_tokens], every row written; a row
+ *                  whose patch id is >= p gets NaN when k > 1.
+ *   pool_size_out: device int32 [n_layers] (may be NULL): k of each layer.
+ * CV is computed in fp32 (two passes: mean, then squared deviations).
+ * Errors: IPV_EINVAL (non-positive sizes, n_tokens above IPV_MAX_TOKENS,
+ * p above IPV_MAX_POOL_FRAME_TOKENS or a grid too large for its bordered map,
+ * id_stride < n_tokens, only one id array,
+ * unordered or NaN thresholds, NULL or misaligned pointers), IPV_ENOINIT,
+ * IPV_ECUDA. */
+ipv_status ipv_van_pool(const float* van, const uint16_t* patch_id, const uint32_t* frame_id,
+                        int64_t id_stride, int n_layers, int n_kv_heads, int64_t n_tokens,
+                        int frame_grid_h, int frame_grid_w, const float cv_tau[3],
+                        float* pooled_out, int32_t* pool_size_out, void* stream);
 
 /* The recent-frame count r the library uses for a cache of n_frames frames
  * (the ipv_init override if set, else max(1, floor(n_frames/8 + 1/2))).
@@ -152,8 +208,8 @@ const char* ipv_status_string(ipv_status s);
 /* Kernel timing for benchmarks: while enabled, ipv_compress and ipv_score
  * record CUDA events around each kernel on the call's stream. Kernel ids:
  * 0 recent-frame mean, 1 scoring, 2 selection, 3 compaction, 4 the
- * single-kernel pass. */
-#define IPV_NUM_KERNELS 5
+ * single-kernel pass, 5 VaN pooling. */
+#define IPV_NUM_KERNELS 6
 ipv_status ipv_profile_enable(int on);
 
 /* Waits (at most timeout_ms) for the recorded events, then writes per kernel

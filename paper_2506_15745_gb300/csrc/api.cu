@@ -11,6 +11,7 @@
 #include "ipv_common.cuh"
 
 static_assert(ipv::kMaxTokens == IPV_MAX_TOKENS, "selection shared-memory limit");
+static_assert(ipv::kMaxPoolFrame == IPV_MAX_POOL_FRAME_TOKENS, "pooling shared-memory limit");
 
 namespace {
 
@@ -25,6 +26,7 @@ struct State {
   float* tar = nullptr;   // [max_slabs][token_capacity]
   float* van = nullptr;
   float* m = nullptr;     // [max_slabs][max_frame_tokens][max_head_dim]
+  float* pooled = nullptr;  // [max_slabs][token_capacity], van_pool only
   ipv::PipeState* pstate = nullptr;
   unsigned* pflags = nullptr;  // [kPipeFlags][max_slabs]
   bool pipe_dirty = false;     // a failed launch may have left queue state behind
@@ -133,7 +135,13 @@ ipv_status check_cache(const ipv_kv* k, const ipv_kv* v, int L, int H, int D, in
     const uint16_t* ps = k->patch_id[k->cur];
     const uint16_t* pd = k->patch_id[1 - k->cur];
     if (pd && pd == ps) return fail(IPV_EINVAL, "patch-id halves must be distinct buffers");
+    const uint32_t* fs = k->frame_id[k->cur];
+    const uint32_t* fd = k->frame_id[1 - k->cur];
+    if (fd && fd == fs) return fail(IPV_EINVAL, "frame-id halves must be distinct buffers");
+    if (fd && (reinterpret_cast<uintptr_t>(fd) & 3u)) return fail(IPV_EINVAL, "frame ids must be 4-byte aligned");
   }
+  const uint32_t* fsrc = k->frame_id[k->cur];
+  if (fsrc && (reinterpret_cast<uintptr_t>(fsrc) & 3u)) return fail(IPV_EINVAL, "frame ids must be 4-byte aligned");
   if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
   const int64_t S = static_cast<int64_t>(L) * H;
   if (S > g.opt.max_slabs)
@@ -210,6 +218,7 @@ void ipv_shutdown(void) {
   cudaFree(g.tar);
   cudaFree(g.van);
   cudaFree(g.m);
+  cudaFree(g.pooled);
   cudaFree(g.pstate);
   cudaFree(g.pflags);
   g = State{};
@@ -228,6 +237,15 @@ ipv_status ipv_init(const ipv_options* opt) {
     return fail(IPV_EINVAL, "token_capacity must be in [1, 2^31)");
   if (opt->single_kernel != 0 && opt->single_kernel != 1)
     return fail(IPV_EINVAL, "single_kernel must be 0 or 1");
+  if (opt->van_pool != 0 && opt->van_pool != 1) return fail(IPV_EINVAL, "van_pool must be 0 or 1");
+  if (opt->van_pool) {
+    if (opt->single_kernel) return fail(IPV_EINVAL, "van_pool runs with the step kernels only (single_kernel = 0)");
+    if (opt->max_frame_tokens > IPV_MAX_POOL_FRAME_TOKENS)
+      return fail(IPV_EINVAL, "van_pool needs max_frame_tokens <= %d", IPV_MAX_POOL_FRAME_TOKENS);
+    const float* t = opt->cv_tau;
+    if (t[0] != t[0] || t[1] != t[1] || t[2] != t[2] || !(t[0] <= t[1] && t[1] <= t[2]))
+      return fail(IPV_EINVAL, "cv_tau must be ordered tau_1 <= tau_2 <= tau_3 (no NaN)");
+  }
   ipv_shutdown();
   int n_dev = 0;
   cudaError_t e = cudaGetDeviceCount(&n_dev);
@@ -241,6 +259,7 @@ ipv_status ipv_init(const ipv_options* opt) {
     return cuda_fail(e, "no usable kernel image for this device (built for sm_103a)");
   if ((e = ipv::select_prepare(IPV_MAX_TOKENS)) != cudaSuccess) return cuda_fail(e, "select kernel set-up");
   if ((e = ipv::pipeline_prepare()) != cudaSuccess) return cuda_fail(e, "pipeline kernel set-up");
+  if ((e = ipv::pool_prepare()) != cudaSuccess) return cuda_fail(e, "pooling kernel set-up");
   State s;
   s.opt = *opt;
   s.num_sms = prop.multiProcessorCount;
@@ -250,21 +269,25 @@ ipv_status ipv_init(const ipv_options* opt) {
   const size_t flag_bytes = ipv::kPipeFlags * static_cast<size_t>(opt->max_slabs) * sizeof(unsigned);
   if (cudaMalloc(&s.tar, score_bytes) != cudaSuccess || cudaMalloc(&s.van, score_bytes) != cudaSuccess ||
       cudaMalloc(&s.m, m_bytes) != cudaSuccess ||
+      (opt->van_pool && cudaMalloc(&s.pooled, score_bytes) != cudaSuccess) ||
       cudaMalloc(&s.pstate, sizeof(ipv::PipeState)) != cudaSuccess ||
       cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess) {
     cudaGetLastError();
     cudaFree(s.tar);
     cudaFree(s.van);
     cudaFree(s.m);
+    cudaFree(s.pooled);
     cudaFree(s.pstate);
     cudaFree(s.pflags);
-    return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated", 2 * score_bytes + m_bytes);
+    return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated",
+                (opt->van_pool ? 3 : 2) * score_bytes + m_bytes);
   }
   if ((e = cudaMemset(s.pstate, 0, sizeof(ipv::PipeState))) != cudaSuccess ||
       (e = cudaMemset(s.pflags, 0, flag_bytes)) != cudaSuccess) {
     cudaFree(s.tar);
     cudaFree(s.van);
     cudaFree(s.m);
+    cudaFree(s.pooled);
     cudaFree(s.pstate);
     cudaFree(s.pflags);
     return cuda_fail(e, "clearing the pipeline state");
@@ -309,6 +332,7 @@ ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_he
   a.tar = tar_out;
   a.van = van_out;
   a.zero_recent = 1;
+  a.van_recent = g.opt.van_pool;
   a.num_sms = g.num_sms;
   a.error = &g.pstate->error;
   prof_begin(0, st);
@@ -378,6 +402,10 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   if (sh.rp >= budget)
     return fail(IPV_EINVAL, "recent tokens r*p = %lld must be below budget %lld", static_cast<long long>(sh.rp),
                 static_cast<long long>(budget));
+  if (g.opt.van_pool && k->patch_id[k->cur] && !k->frame_id[k->cur])
+    return fail(IPV_EINVAL, "pooled VaN needs frame ids for a cache with patch ids");
+  if (g.opt.van_pool && ipv::pool_smem_bytes(frame_grid_h, frame_grid_w, true) == 0)
+    return fail(IPV_EINVAL, "frame too large for pooled VaN");
 
   ipv::ScoreArgs a{};
   a.k = k->buf[k->cur];
@@ -394,12 +422,13 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   a.tar = g.tar;
   a.van = g.van;
   a.zero_recent = 0;
+  a.van_recent = g.opt.van_pool;
   a.num_sms = g.num_sms;
   a.error = &g.pstate->error;
 
   ipv::SelectArgs sa{};
   sa.tar = g.tar;
-  sa.van = g.van;
+  sa.van = g.opt.van_pool ? g.pooled : g.van;
   sa.n_slabs = sh.S;
   sa.n_tokens = sh.N;
   sa.rp = sh.rp;
@@ -414,6 +443,8 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   ga.v_dst = v->buf[1 - v->cur];
   ga.pid_src = k->patch_id[k->cur];
   ga.pid_dst = k->patch_id[1 - k->cur];
+  ga.fid_src = k->frame_id[k->cur];
+  ga.fid_dst = k->frame_id[1 - k->cur];
   ga.kept = kept_idx_out;
   ga.n_slabs = sh.S;
   ga.cap = g.opt.token_capacity;
@@ -477,6 +508,25 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   e = ipv::launch_score(a, st);
   prof_end(1, st);
   if (e != cudaSuccess) return cuda_fail(e, "scoring kernel");
+  if (g.opt.van_pool) {  // the VaN stage ranks layer-adaptive pooled VaN
+    ipv::PoolArgs pa{};
+    pa.van = g.van;
+    pa.pooled = g.pooled;
+    pa.patch_id = k->patch_id[k->cur];
+    pa.frame_id = pa.patch_id ? k->frame_id[k->cur] : nullptr;
+    pa.id_stride = g.opt.token_capacity;
+    pa.n_slabs = sh.S;
+    pa.n_tokens = sh.N;
+    pa.n_rows = sh.N - sh.rp;
+    pa.n_heads = n_kv_heads;
+    pa.grid_h = frame_grid_h;
+    pa.grid_w = frame_grid_w;
+    for (int i = 0; i < 3; ++i) pa.tau[i] = g.opt.cv_tau[i];
+    prof_begin(5, st);
+    e = ipv::launch_pool(pa, st, true);
+    prof_end(5, st);
+    if (e != cudaSuccess) return cuda_fail(e, "VaN pooling kernel");
+  }
   prof_begin(2, st);
   e = ipv::launch_select(sa, st);
   prof_end(2, st);
@@ -489,6 +539,51 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   k->cur = 1 - k->cur;
   v->cur = 1 - v->cur;
   return IPV_OK;
+}
+
+ipv_status ipv_van_pool(const float* van, const uint16_t* patch_id, const uint32_t* frame_id,
+                        int64_t id_stride, int n_layers, int n_kv_heads, int64_t n_tokens,
+                        int frame_grid_h, int frame_grid_w, const float cv_tau[3],
+                        float* pooled_out, int32_t* pool_size_out, void* stream) {
+  if (!van || !pooled_out || !cv_tau) return fail(IPV_EINVAL, "van, pooled_out and cv_tau must not be NULL");
+  if ((reinterpret_cast<uintptr_t>(van) & 3u) || (reinterpret_cast<uintptr_t>(pooled_out) & 3u) ||
+      (reinterpret_cast<uintptr_t>(pool_size_out) & 3u) || (reinterpret_cast<uintptr_t>(frame_id) & 3u) ||
+      (reinterpret_cast<uintptr_t>(patch_id) & 1u))
+    return fail(IPV_EINVAL, "misaligned pointer");
+  if (n_layers <= 0 || n_kv_heads <= 0 || n_tokens <= 0 || frame_grid_h <= 0 || frame_grid_w <= 0)
+    return fail(IPV_EINVAL, "sizes must be positive");
+  if (n_tokens > IPV_MAX_TOKENS) return fail(IPV_EINVAL, "n_tokens exceeds IPV_MAX_TOKENS");
+  const int64_t p = static_cast<int64_t>(frame_grid_h) * frame_grid_w;
+  if (p > IPV_MAX_POOL_FRAME_TOKENS)
+    return fail(IPV_EINVAL, "frame of %lld tokens exceeds IPV_MAX_POOL_FRAME_TOKENS", static_cast<long long>(p));
+  if (ipv::pool_smem_bytes(frame_grid_h, frame_grid_w, true) == 0) return fail(IPV_EINVAL, "frame too large for pooled VaN");
+  if ((patch_id == nullptr) != (frame_id == nullptr))
+    return fail(IPV_EINVAL, "patch_id and frame_id must both be set or both be NULL");
+  if (patch_id && id_stride < n_tokens) return fail(IPV_EINVAL, "id_stride is below n_tokens");
+  const float* t = cv_tau;
+  if (t[0] != t[0] || t[1] != t[1] || t[2] != t[2] || !(t[0] <= t[1] && t[1] <= t[2]))
+    return fail(IPV_EINVAL, "cv_tau must be ordered tau_1 <= tau_2 <= tau_3 (no NaN)");
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  cudaSetDevice(g.opt.device);
+  ipv::PoolArgs pa{};
+  pa.van = van;
+  pa.pooled = pooled_out;
+  pa.pool_size = pool_size_out;
+  pa.patch_id = patch_id;
+  pa.frame_id = frame_id;
+  pa.id_stride = id_stride;
+  pa.n_slabs = static_cast<int64_t>(n_layers) * n_kv_heads;
+  pa.n_tokens = n_tokens;
+  pa.n_rows = n_tokens;
+  pa.n_heads = n_kv_heads;
+  pa.grid_h = frame_grid_h;
+  pa.grid_w = frame_grid_w;
+  for (int i = 0; i < 3; ++i) pa.tau[i] = t[i];
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  prof_begin(5, st);
+  cudaError_t e = ipv::launch_pool(pa, st, false);
+  prof_end(5, st);
+  return after_launch(e, "VaN pooling kernel");
 }
 
 ipv_status ipv_device_error(uint32_t* err_out) {

@@ -7,8 +7,8 @@
 //
 // Pure data movement (HBM-bound): a half-warp moves one 16-byte-chunked K row
 // and the matching V row; the flattened (slab, j) space is strided over the
-// whole grid with several rows in flight per half-warp. Patch ids travel with
-// their rows.
+// whole grid with several rows in flight per half-warp. Patch and frame ids
+// travel with their rows, copied by a separate coalesced loop.
 #include "pass_device.cuh"
 
 namespace ipv {
@@ -21,7 +21,8 @@ __global__ void __launch_bounds__(512, 2) gather_kernel(GatherArgs a) {
   constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
   const int64_t n_hw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
   const int64_t hw = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 4;
-  dev::gather_range<CPL, kU, true>(a, 0, a.n_slabs * a.budget, hw, n_hw);
+  dev::gather_ids(a);
+  dev::gather_range<CPL, kU, true, false>(a, 0, a.n_slabs * a.budget, hw, n_hw);
 }
 
 template <int CPL>

@@ -167,7 +167,8 @@ struct ScoreArgs {
   float* m;                 // scratch [S][p][D] fp32
   float* tar;               // [S][n_tokens]
   float* van;
-  int zero_recent;          // write 0 to the recent-frame entries of tar/van
+  int zero_recent;          // write 0 to the recent-frame entries of tar (and van unless van_recent)
+  int van_recent;           // write the VaN of the recent rows to van (pooled VaN's CV counts them)
   int num_sms;
   unsigned* error;          // device word: bit 2 set if a bulk-copy wait timed out
 };
@@ -211,6 +212,8 @@ struct GatherArgs {
   void* v_dst;
   const uint16_t* pid_src;  // nullptr: patch = n mod p
   uint16_t* pid_dst;        // nullptr: not written
+  const uint32_t* fid_src;  // nullptr: frame = n div p
+  uint32_t* fid_dst;        // nullptr: not written
   const int32_t* kept;      // [S][budget]
   int64_t n_slabs, cap, budget;
   int row_bytes, p;
@@ -219,6 +222,24 @@ struct GatherArgs {
 
 int gather_cpl(int row_bytes);  // 16-byte chunks per lane of a half-warp row copy
 cudaError_t launch_gather(const GatherArgs& a, cudaStream_t st);
+
+// Layer-adaptive pooling of VaN (pool.cu): one block per slab.
+constexpr int kPoolThreads = 1024;
+constexpr int kMaxPoolFrame = 4096;  // IPV_MAX_POOL_FRAME_TOKENS
+struct PoolArgs {
+  const float* van;          // [S][n_tokens] VaN of every cached row
+  float* pooled;             // [S][n_tokens]: rows [0, n_rows) written
+  int32_t* pool_size;        // [S / n_heads] or nullptr
+  const uint16_t* patch_id;  // [S][id_stride] or nullptr (then frame_id is nullptr too)
+  const uint32_t* frame_id;
+  int64_t id_stride;
+  int64_t n_slabs, n_tokens, n_rows;
+  int n_heads, grid_h, grid_w;
+  float tau[3];
+};
+size_t pool_smem_bytes(int grid_h, int grid_w, bool staged);  // 0 if a frame does not fit
+cudaError_t pool_prepare();
+cudaError_t launch_pool(const PoolArgs& a, cudaStream_t st, bool pdl);
 
 // Single-kernel pass (pipeline.cu). The queue state lives in library scratch,
 // is zero before a launch and is reset by the kernel's last block.

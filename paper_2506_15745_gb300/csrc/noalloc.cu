@@ -129,6 +129,9 @@ extern "C" ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype,
   const uint16_t* pid_src = k->patch_id[k->cur];
   uint16_t* pid_dst = k->patch_id[1 - k->cur];
   if (evict && pid_dst && pid_dst == pid_src) return reject(IPV_EINVAL, "patch-id halves must be distinct");
+  if (evict && (!aligned(k->frame_id[0], 4) || !aligned(k->frame_id[1], 4) ||
+                (k->frame_id[1 - k->cur] && k->frame_id[1 - k->cur] == k->frame_id[k->cur])))
+    return reject(IPV_EINVAL, "frame-id halves must be distinct and 4-byte aligned");
   const int64_t S = static_cast<int64_t>(n_layers) * n_kv_heads;
   const int64_t f = n_tokens / p;
   int r = recent_frames;
@@ -205,6 +208,8 @@ extern "C" ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype,
   ga.v_dst = vd;
   ga.pid_src = pid_src;
   ga.pid_dst = pid_dst;
+  ga.fid_src = k->frame_id[k->cur];
+  ga.fid_dst = k->frame_id[1 - k->cur];
   ga.kept = kept_idx_out;
   ga.n_slabs = S;
   ga.cap = token_capacity;

@@ -73,6 +73,36 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
         for (int e = 0; e < P2; ++e) acc[i][e] = fma2(x[i][e], inv2, acc[i][e]);
     }
   }
+  if (a.van_recent) {  // VaN of the r recent rows of patch q (Sec. 3.2), for a layer's CV
+    const char* vslab = static_cast<const char*>(a.v) + s * a.cap * row_bytes;
+    for (int t0 = 0; t0 < a.r; t0 += kBatch) {  // uniform across the warp
+      uint4 raw[kBatch][CPL];
+#pragma unroll
+      for (int b = 0; b < kBatch; ++b) {
+        const bool ok = col_ok && t0 + b < a.r;
+        const char* row = vslab + (n_past + static_cast<int64_t>(t0 + b) * a.p + q) * row_bytes;
+#pragma unroll
+        for (int i = 0; i < CPL; ++i) {
+          const int c = sub + LPR * i;
+          raw[b][i] = (ok && c < n_chunks) ? ld_stream(row + c * 16) : make_uint4(0, 0, 0, 0);
+        }
+      }
+#pragma unroll
+      for (int b = 0; b < kBatch; ++b) {
+        float2 vv2 = make_float2(0.0f, 0.0f);
+#pragma unroll
+        for (int i = 0; i < CPL; ++i) {
+          float2 x[P2];
+          Chunk<T>::widen2(raw[b][i], x);
+#pragma unroll
+          for (int e = 0; e < P2; ++e) vv2 = fma2(x[e], x[e], vv2);
+        }
+        const float vv = group_sum<LPR>(vv2.x + vv2.y);
+        if (col_ok && sub == 0 && t0 + b < a.r)
+          a.van[s * a.n_tokens + n_past + static_cast<int64_t>(t0 + b) * a.p + q] = sqrtf(vv);
+      }
+    }
+  }
   if (!col_ok) return;
   const float inv_r = 1.0f / static_cast<float>(a.r);
   float* mrow = a.m + (s * a.p + q) * static_cast<int64_t>(a.D);
@@ -91,9 +121,10 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
     for (int t = 0; t < a.r; ++t) {
       const int64_t n = n_past + static_cast<int64_t>(t) * a.p + q;
       a.tar[s * a.n_tokens + n] = 0.0f;
-      a.van[s * a.n_tokens + n] = 0.0f;
+      if (!a.van_recent) a.van[s * a.n_tokens + n] = 0.0f;
     }
   }
+
 }
 
 // Where score_segment reads the m table from.
@@ -807,8 +838,9 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
 // Half-warp hw (of n_hw) copies rows g = g_begin + hw, g_begin + hw + n_hw,
 // ... of the flattened (slab, j) range [g_begin, g_end), kU rows in flight.
 // Kept indices and source patch ids are read with plain loads (the kept
-// indices may have been written earlier in the same kernel).
-template <int CPL, int kU, bool REVERSE = false>
+// indices may have been written earlier in the same kernel). IDS: copy the
+// patch and frame ids of each row here too (else gather_ids does it).
+template <int CPL, int kU, bool REVERSE = false, bool IDS = true>
 __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begin, int64_t g_end,
                                              int64_t hw, int64_t n_hw) {
   const int lane = threadIdx.x & 15;
@@ -858,7 +890,7 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
           st_stream(vd + dst_off[u] + ch * 16, vr[u][c]);
         }
       }
-      if (a.pid_dst && lane == 0) {
+      if (IDS && a.pid_dst && lane == 0) {
         const int64_t t = g0 + u * n_hw;
         const int64_t g = REVERSE ? g_end - 1 - (t - g_begin) : t;
         const int64_t s = g / a.budget;
@@ -866,7 +898,34 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
         a.pid_dst[s * a.cap + j] = a.pid_src ? a.pid_src[s * a.cap + src_n[u]]
                                              : static_cast<uint16_t>(src_n[u] % a.p);
       }
+      if (IDS && a.fid_dst && lane == 1) {  // frame ids travel with their rows too
+        const int64_t t = g0 + u * n_hw;
+        const int64_t g = REVERSE ? g_end - 1 - (t - g_begin) : t;
+        const int64_t s = g / a.budget;
+        const int64_t j = g - s * a.budget;
+        a.fid_dst[s * a.cap + j] = a.fid_src ? a.fid_src[s * a.cap + src_n[u]]
+                                             : static_cast<uint32_t>(src_n[u] / a.p);
+      }
     }
+  }
+}
+
+// Patch and frame ids of the kept rows, one (slab, j) per thread of the
+// grid: consecutive j of a slab are consecutive threads, so the stores are
+// coalesced (ids travel with their rows, Sec. 3.1 K~ = K[:, I, :]).
+__device__ __forceinline__ void gather_ids(const GatherArgs& a) {
+  if (!a.pid_dst && !a.fid_dst) return;
+  const int64_t total = a.n_slabs * a.budget;
+  const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total; g += step) {
+    const int n = a.kept[g];
+    if (n < 0 || n >= a.cap) continue;
+    const int64_t s = g / a.budget;
+    const int64_t dst = s * a.cap + (g - s * a.budget);
+    if (a.pid_dst)
+      a.pid_dst[dst] = a.pid_src ? a.pid_src[s * a.cap + n] : static_cast<uint16_t>(n % a.p);
+    if (a.fid_dst)
+      a.fid_dst[dst] = a.fid_src ? a.fid_src[s * a.cap + n] : static_cast<uint32_t>(n / a.p);
   }
 }
 

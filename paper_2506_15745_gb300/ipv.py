@@ -15,9 +15,10 @@ LIB_PATH = os.path.join(_HERE, "libipv.so")
 
 IPV_OK, IPV_EINVAL, IPV_ENOINIT, IPV_ENOMEM, IPV_ECUDA, IPV_ETIMEOUT = range(6)
 IPV_BF16, IPV_F32 = 0, 1
-NUM_KERNELS = 5
-KERNEL_NAMES = ("recent_mean", "score", "select", "gather", "pipeline")
+NUM_KERNELS = 6
+KERNEL_NAMES = ("recent_mean", "score", "select", "gather", "pipeline", "pool")
 MAX_TOKENS = 49152
+MAX_POOL_FRAME_TOKENS = 4096
 
 
 class IpvError(RuntimeError):
@@ -30,20 +31,23 @@ class Options(ctypes.Structure):
     _fields_ = [("device", ctypes.c_int), ("dtype", ctypes.c_int),
                 ("recent_frames", ctypes.c_int), ("max_head_dim", ctypes.c_int),
                 ("max_frame_tokens", ctypes.c_int), ("max_slabs", ctypes.c_int64),
-                ("token_capacity", ctypes.c_int64), ("single_kernel", ctypes.c_int)]
+                ("token_capacity", ctypes.c_int64), ("single_kernel", ctypes.c_int),
+                ("van_pool", ctypes.c_int), ("cv_tau", ctypes.c_float * 3)]
 
 
 class KV(ctypes.Structure):
     """ipv_kv: the two halves of one ping-pong cache tensor (K or V)."""
     _fields_ = [("buf", ctypes.c_void_p * 2), ("patch_id", ctypes.c_void_p * 2),
-                ("cur", ctypes.c_int)]
+                ("cur", ctypes.c_int), ("frame_id", ctypes.c_void_p * 2)]
 
     @classmethod
-    def from_tensors(cls, halves, patch_ids=(None, None), cur: int = 0) -> "KV":
+    def from_tensors(cls, halves, patch_ids=(None, None), cur: int = 0,
+                     frame_ids=(None, None)) -> "KV":
         kv = cls()
         for h in range(2):
             kv.buf[h] = _ptr(halves[h])
             kv.patch_id[h] = _ptr(patch_ids[h])
+            kv.frame_id[h] = _ptr(frame_ids[h])
         kv.cur = cur
         return kv
 
@@ -87,9 +91,11 @@ def load():
         lib.ipv_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32)]
         lib.ipv_compress_static.argtypes = [KVP, KVP, I32, I64, I32, I32, I32, I32, I64, I32, I32,
                                             I64, F, P, P]
+        lib.ipv_van_pool.argtypes = [P, P, P, I64, I32, I32, I64, I32, I32,
+                                     ctypes.POINTER(ctypes.c_float), P, P, P]
         for name in ("ipv_init", "ipv_compress", "ipv_score", "ipv_select",
                      "ipv_profile_enable", "ipv_profile_collect", "ipv_device_error",
-                     "ipv_compress_static"):
+                     "ipv_compress_static", "ipv_van_pool"):
             getattr(lib, name).restype = I32
         _lib = lib
     return _lib
@@ -113,9 +119,13 @@ def last_error() -> str:
 
 def init(*, device: int = 0, dtype: str = "bf16", recent_frames: int = 0, max_head_dim: int,
          max_frame_tokens: int, max_slabs: int, token_capacity: int,
-         single_kernel: bool = False) -> None:
+         single_kernel: bool = False, van_pool: bool = False,
+         cv_tau=(0.0, 0.0, 0.0)) -> None:
+    """ipv_init. van_pool: the VaN stage ranks layer-adaptive pooled VaN with
+    pool size g(CV) from the thresholds cv_tau (Sec. 3.2, Algorithm 2)."""
     opt = Options(device, IPV_BF16 if dtype == "bf16" else IPV_F32, recent_frames, max_head_dim,
-                  max_frame_tokens, max_slabs, token_capacity, int(bool(single_kernel)))
+                  max_frame_tokens, max_slabs, token_capacity, int(bool(single_kernel)),
+                  int(bool(van_pool)), (ctypes.c_float * 3)(*[float(t) for t in cv_tau]))
     _check(load().ipv_init(ctypes.byref(opt)))
 
 
@@ -163,6 +173,16 @@ def select(tar, van, n_slabs: int, n_tokens: int, frame_grid_h: int, frame_grid_
            budget: int, tar_ratio: float, kept_idx_out, stream=None) -> None:
     _check(load().ipv_select(_ptr(tar), _ptr(van), n_slabs, n_tokens, frame_grid_h, frame_grid_w,
                              budget, tar_ratio, _ptr(kept_idx_out), _stream(stream)))
+
+
+def van_pool(van, n_layers: int, n_kv_heads: int, n_tokens: int, frame_grid_h: int,
+             frame_grid_w: int, cv_tau, pooled_out, pool_size_out=None, patch_id=None,
+             frame_id=None, id_stride: int = 0, stream=None) -> None:
+    """ipv_van_pool: layer-adaptive pooled VaN of every row (and each layer's pool size)."""
+    tau = (ctypes.c_float * 3)(*[float(t) for t in cv_tau])
+    _check(load().ipv_van_pool(_ptr(van), _ptr(patch_id), _ptr(frame_id), id_stride, n_layers,
+                               n_kv_heads, n_tokens, frame_grid_h, frame_grid_w, tau,
+                               _ptr(pooled_out), _ptr(pool_size_out), _stream(stream)))
 
 
 def device_error() -> int:

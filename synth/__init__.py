@@ -111,6 +111,11 @@ CONFIGS = {
     "llava_pool": Workload("llava_pool", 28, 4, 128, "bf16", 14, 14, 48, 6272, 0.5,
                            value_sigma=0.25, value_sigma_last=1.0, value_locality=0.9,
                            van_pool=True, cv_tau=(0.4, 0.6, 0.9)),
+    # the pooled workload streamed like "stream" (frame ids travel with the rows)
+    "stream_pool": Workload("stream_pool", 28, 4, 128, "bf16", 14, 14, 48, 6272, 0.5,
+                            value_sigma=0.25, value_sigma_last=1.0, value_locality=0.9,
+                            van_pool=True, cv_tau=(0.4, 0.6, 0.9),
+                            stream_frames=3600, append_frames=16),
 }
 
 

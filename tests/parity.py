@@ -107,3 +107,39 @@ def assert_gather_exact(src, dst, kept, budget):
     for s in range(S):
         idx = kept[s]
         assert np.array_equal(dst[s, :budget], src[s, idx]), f"slab {s}: compacted rows differ"
+
+
+INF = float("inf")
+FORCE_POOL = {7: (INF, INF, INF), 5: (0.0, INF, INF), 3: (0.0, 0.0, INF), 1: (0.0, 0.0, 0.0)}
+
+
+def pooled_reference(van_all_o, n_heads, gh, gw, tau, ks_gpu, pid=None, fid=None):
+    """Oracle pooled VaN for layer-adaptive pooling, checked against the GPU's
+    per-layer pool sizes. The pool size is an integer decided by a floating
+    CV: it must equal the oracle's, except where the oracle's CV lies within
+    TOL (relative) of a threshold; there the GPU's size is accepted and the
+    oracle pools with it. Returns (pooled [S, N], oracle sizes, oracle CVs)."""
+    pooled, ks, cv = oracle.van_pool(van_all_o, n_heads, gh, gw, tau, pid, fid)
+    for layer in range(len(ks)):
+        kg = int(ks_gpu[layer])
+        if kg == ks[layer]:
+            continue
+        near = any(abs(cv[layer] - t) <= TOL * max(abs(t), 1e-30) for t in tau)
+        assert near, f"layer {layer}: pool size {kg} vs oracle {ks[layer]} (CV {cv[layer]:.9g})"
+        sl = slice(layer * n_heads, (layer + 1) * n_heads)
+        sub_p = None if pid is None else pid[sl]
+        sub_f = None if fid is None else fid[sl]
+        pooled[sl] = oracle.van_pool(van_all_o[sl], n_heads, gh, gw, FORCE_POOL[kg], sub_p, sub_f)[0]
+    return pooled, ks, cv
+
+
+def assert_pooled_close(g, o, rows=None):
+    """Pooled VaN: |g - o| <= TOL |o| (NaN exactly where the oracle has NaN)."""
+    g = np.asarray(g, np.float64)
+    if rows is not None:
+        g, o = g[:, :rows], o[:, :rows]
+    nan_o = np.isnan(o)
+    assert np.array_equal(np.isnan(g), nan_o), "NaN positions differ"
+    err = np.abs(g - o)[~nan_o] / np.maximum(np.abs(o[~nan_o]), 1e-30)
+    assert err.max(initial=0.0) <= TOL, f"pooled VaN error {err.max():.3g}"
+    return float(err.max(initial=0.0))

@@ -79,9 +79,45 @@ def test_init_option_checks(lib):
     good = dict(device=0, dtype=0, recent_frames=0, max_head_dim=128, max_frame_tokens=196,
                 max_slabs=112, token_capacity=9408)
     for key, bad in [("dtype", 7), ("max_head_dim", 1024), ("max_frame_tokens", 0),
-                     ("max_slabs", 0), ("token_capacity", -1), ("recent_frames", -1), ("device", -1)]:
+                     ("max_slabs", 0), ("token_capacity", -1), ("recent_frames", -1), ("device", -1),
+                     ("van_pool", 2)]:
         opt = ipv.Options(**dict(good, **{key: bad}))
         assert lib.ipv_init(ctypes.byref(opt)) == ipv.IPV_EINVAL, key
+    tau = lambda *t: (ctypes.c_float * 3)(*t)  # noqa: E731
+    pooled = dict(good, van_pool=1, cv_tau=tau(0.4, 0.6, 0.9))
+    for key, bad in [("single_kernel", 1), ("max_frame_tokens", ipv.MAX_POOL_FRAME_TOKENS + 1),
+                     ("cv_tau", tau(0.6, 0.4, 0.9)), ("cv_tau", tau(0.4, float("nan"), 0.9))]:
+        opt = ipv.Options(**dict(pooled, **{key: bad}))
+        assert lib.ipv_init(ctypes.byref(opt)) == ipv.IPV_EINVAL, key
+
+
+def test_van_pool_host_checks(lib):
+    tau = (ctypes.c_float * 3)(0.4, 0.6, 0.9)
+    call = lambda **kw: lib.ipv_van_pool(  # noqa: E731
+        kw.get("van", 0x1000), kw.get("pid", None), kw.get("fid", None), kw.get("stride", 0),
+        kw.get("L", 28), kw.get("H", 4), kw.get("N", 9408), kw.get("gh", 14), kw.get("gw", 14),
+        kw.get("tau", tau), kw.get("out", 0x2000), kw.get("ks", None), None)
+    assert call(van=None) == ipv.IPV_EINVAL
+    assert call(out=0x2002) == ipv.IPV_EINVAL                   # misaligned
+    assert call(N=0) == ipv.IPV_EINVAL
+    assert call(N=ipv.MAX_TOKENS + 1) == ipv.IPV_EINVAL
+    assert call(gh=65, gw=64) == ipv.IPV_EINVAL                 # frame above the pooling limit
+    assert call(gh=1, gw=4096) == ipv.IPV_EINVAL                # bordered map too large
+    assert call(pid=0x3000) == ipv.IPV_EINVAL                   # patch ids without frame ids
+    assert call(pid=0x3000, fid=0x4000, stride=9407) == ipv.IPV_EINVAL
+    assert call(tau=(ctypes.c_float * 3)(0.9, 0.6, 0.4)) == ipv.IPV_EINVAL
+    assert call(pid=0x3000, fid=0x4000, stride=9408) == ipv.IPV_ENOINIT
+    assert call() == ipv.IPV_ENOINIT
+
+
+def test_frame_id_checks(lib):
+    k = ipv.KV.from_tensors((0x1000, 0x2000), (None, None), 0, (0x5000, 0x5000))
+    v = _kv((0x3000, 0x4000))
+    assert lib.ipv_compress(ctypes.byref(k), ctypes.byref(v), 28, 4, 128, 9408, 14, 14, 6272, 0.5,
+                            0x6000, None) == ipv.IPV_EINVAL    # aliasing frame-id halves
+    k = ipv.KV.from_tensors((0x1000, 0x2000), (None, None), 0, (0x5000, 0x5002))
+    assert lib.ipv_compress(ctypes.byref(k), ctypes.byref(v), 28, 4, 128, 9408, 14, 14, 6272, 0.5,
+                            0x6000, None) == ipv.IPV_EINVAL    # misaligned frame ids
 
 
 def test_init_without_gpu_fails_cleanly(lib):
