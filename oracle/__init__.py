@@ -13,6 +13,9 @@ Functions mirror the paper's steps:
   van_all(), pool_size(), van_pool(), compress_pooled()
             -- layer-adaptive VaN pooling (Sec. 3.2, Algorithm 2) and the pass
                whose VaN stage ranks pooled VaN
+  scores_shared(), van_all_shared(), compress_shared()
+            -- one index set per layer shared by its KV heads (Sec. 3.1,
+               K~ = K[:, I, :]): scores of the concatenated H x D blocks
 """
 from __future__ import annotations
 
@@ -64,7 +67,11 @@ def _load():
         lib.oracle_gather_patch.argtypes = [P, P, I64, I64, I64, I32, P, I64]
         lib.oracle_gather_patch.restype = I32
         lib.oracle_compress.argtypes = [P, P, I32, I64, I64, I32, I64, I32, I32, I64, D,
-                                        P, P, P, P, P, I32, P, I32, I32, P, P, P]
+                                        P, P, P, P, P, I32, P, I32, I32, P, P, P, I32]
+        lib.oracle_scores_shared.argtypes = [P, P, I32, I64, I32, I64, I32, I64, I32, I32, P, P, P]
+        lib.oracle_scores_shared.restype = I32
+        lib.oracle_van_all_shared.argtypes = [P, I32, I64, I32, I64, I32, I64, P]
+        lib.oracle_van_all_shared.restype = I32
         lib.oracle_compress.restype = I32
         lib.oracle_gather_frame.argtypes = [P, P, I64, I64, I64, I32, P, I64]
         lib.oracle_gather_frame.restype = I32
@@ -186,7 +193,7 @@ def compress(k: np.ndarray, v: np.ndarray, n_tokens: int, p: int, r: int, budget
         patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
     rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
                                  budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
-                                 _ptr(pd), _ptr(kept), 0, None, 1, 0, None, None, None)
+                                 _ptr(pd), _ptr(kept), 0, None, 1, 0, None, None, None, 0)
     if rc != 0:
         raise ValueError("oracle_compress rejected its arguments")
     return kept, kd, vd, pd
@@ -257,7 +264,67 @@ def compress_pooled(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, gr
     rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
                                  budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
                                  _ptr(pd), _ptr(kept), 1, _ptr(_tau(tau)), n_kv_heads,
-                                 grid_w, _ptr(frame_id), _ptr(fd), _ptr(ks))
+                                 grid_w, _ptr(frame_id), _ptr(fd), _ptr(ks), 0)
+    if rc != 0:
+        raise ValueError("oracle_compress rejected its arguments")
+    return kept, kd, vd, pd, fd, ks
+
+
+def scores_shared(k: np.ndarray, v: np.ndarray, n_kv_heads: int, n_tokens: int, p: int, r: int,
+                  patch_id: np.ndarray | None = None):
+    """TaR, VaN [L, n_tokens] of the concatenated H x D head blocks of each layer."""
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    S, cap, D = k.shape
+    L = S // n_kv_heads
+    if patch_id is not None:
+        patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
+    tar = np.empty((L, n_tokens), np.float64)
+    van = np.empty((L, n_tokens), np.float64)
+    rc = _load().oracle_scores_shared(_ptr(k), _ptr(v), _kv_kind(k), L, n_kv_heads, cap, D,
+                                      n_tokens, p, r, _ptr(patch_id), _ptr(tar), _ptr(van))
+    if rc != 0:
+        raise ValueError("oracle_scores_shared rejected its arguments")
+    return tar, van
+
+
+def van_all_shared(v: np.ndarray, n_kv_heads: int, n_tokens: int) -> np.ndarray:
+    """Norm of the concatenated H x D value block of every row of every layer."""
+    v = np.ascontiguousarray(v)
+    S, cap, D = v.shape
+    L = S // n_kv_heads
+    out = np.empty((L, n_tokens), np.float64)
+    if _load().oracle_van_all_shared(_ptr(v), _kv_kind(v), L, n_kv_heads, cap, D, n_tokens,
+                                     _ptr(out)) != 0:
+        raise ValueError("oracle_van_all_shared rejected its arguments")
+    return out
+
+
+def compress_shared(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, grid_w: int, r: int,
+                    budget: int, alpha: float, n_kv_heads: int, patch_id=None, frame_id=None,
+                    tau=None):
+    """Whole pass with one index set per layer. Returns (kept [L, budget],
+    K~, V~, patch ids, frame ids, pool size per layer); tau given: pooled VaN."""
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    S, cap, D = k.shape
+    p = grid_h * grid_w
+    L = S // n_kv_heads
+    kd, vd = np.zeros_like(k), np.zeros_like(v)
+    pd = np.zeros((S, cap), np.uint16)
+    fd = np.zeros((S, cap), np.uint32)
+    kept = np.empty((L, budget), np.int32)
+    ks = np.zeros(L, np.int32)
+    if patch_id is not None:
+        patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
+    if frame_id is not None:
+        frame_id = np.ascontiguousarray(frame_id, dtype=np.uint32)
+    pooled = tau is not None
+    rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
+                                 budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
+                                 _ptr(pd), _ptr(kept), int(pooled),
+                                 _ptr(_tau(tau)) if pooled else None, n_kv_heads, grid_w,
+                                 _ptr(frame_id), _ptr(fd), _ptr(ks), 1)
     if rc != 0:
         raise ValueError("oracle_compress rejected its arguments")
     return kept, kd, vd, pd, fd, ks

@@ -44,6 +44,14 @@
 // pooled values. Where rows carry patch ids they also carry frame ids (the
 // frame each token came from); a never-compacted cache has frame n div p.
 //
+// Per-layer shared index set (Sec. 3.1: K is H x N x D and the compressed
+// cache is K[:, I, :], one index set I for all H heads of a layer; likewise
+// Algorithm 2's I_l and J_l per layer), used when the pass is asked for it:
+// a token's key and value are its H x D blocks, the cosine of Eq. (tar) is
+// the l2-normalised (Frobenius) cosine of the concatenated H*D vectors, and
+// VaN is their Frobenius norm. Selection then runs once per layer and every
+// head of the layer is compacted with that layer's indices.
+//
 // Element types: bf16 (widened exactly: bits << 16) or fp32, widened to double.
 
 #include <algorithm>
@@ -146,6 +154,67 @@ int oracle_scores(const void* k, const void* v, int is_bf16, int64_t n_slabs,
       van[n] = l2norm(vv);
     }
   }
+  return 0;
+}
+
+// The H head-rows of token n of layer l, concatenated: slabs l*H .. l*H+H-1.
+static void load_token(const void* base, int is_bf16, int64_t l, int H, int64_t cap, int D, int64_t n,
+                std::vector<double>& out) {
+  out.resize(static_cast<size_t>(H) * D);
+  std::vector<double> row;
+  for (int h = 0; h < H; ++h) {
+    load_row(base, is_bf16, l * H + h, cap, D, n, row);
+    for (int d = 0; d < D; ++d) out[static_cast<size_t>(h) * D + d] = row[d];
+  }
+}
+
+// TaR and VaN of every past token of every layer with one index set per
+// layer (Sec. 3.1, K in R^{H x N x D}): Eq. (tar) on the concatenated H*D key
+// blocks, VaN the norm of the concatenated value block. k, v: [n_layers*H]
+// [cap][D]; patch_id: [n_layers*H][cap] or NULL (the layer's first head's ids
+// are used). tar_out, van_out: [n_layers][n_tokens], recent entries 0.
+int oracle_scores_shared(const void* k, const void* v, int is_bf16, int64_t n_layers, int H,
+                         int64_t cap, int D, int64_t n_tokens, int p, int r,
+                         const uint16_t* patch_id, double* tar_out, double* van_out) {
+  if (!k || !v || !tar_out || !van_out || n_layers < 0 || H <= 0 || D <= 0 || p <= 0 ||
+      r <= 0 || n_tokens < 0 || n_tokens > cap || n_tokens % p != 0)
+    return -1;
+  const int64_t rp = static_cast<int64_t>(r) * p;
+  if (rp > n_tokens) return -1;
+  const int64_t n_past = n_tokens - rp;
+  std::vector<double> kp, kr, vv;
+  for (int64_t l = 0; l < n_layers; ++l) {
+    double* tar = tar_out + l * n_tokens;
+    double* van = van_out + l * n_tokens;
+    for (int64_t n = 0; n < n_tokens; ++n) tar[n] = van[n] = 0.0;
+    for (int64_t n = 0; n < n_past; ++n) {
+      const int64_t q = patch_id ? patch_id[l * H * cap + n] : n % p;
+      if (q < 0 || q >= p) return -1;
+      load_token(k, is_bf16, l, H, cap, D, n, kp);
+      double sum_cos = 0.0;
+      for (int t = 0; t < r; ++t) {
+        load_token(k, is_bf16, l, H, cap, D, n_past + static_cast<int64_t>(t) * p + q, kr);
+        sum_cos += cosine(kp, kr);
+      }
+      tar[n] = -sum_cos / r;
+      load_token(v, is_bf16, l, H, cap, D, n, vv);
+      van[n] = l2norm(vv);
+    }
+  }
+  return 0;
+}
+
+// VaN of every cached row of every layer, shared index set (the norm of the
+// concatenated H x D value block). van_out: [n_layers][n_tokens].
+int oracle_van_all_shared(const void* v, int is_bf16, int64_t n_layers, int H, int64_t cap, int D,
+                          int64_t n_tokens, double* van_out) {
+  if (!v || !van_out || n_layers < 0 || H <= 0 || D <= 0 || n_tokens < 0 || n_tokens > cap) return -1;
+  std::vector<double> vv;
+  for (int64_t l = 0; l < n_layers; ++l)
+    for (int64_t n = 0; n < n_tokens; ++n) {
+      load_token(v, is_bf16, l, H, cap, D, n, vv);
+      van_out[l * n_tokens + n] = l2norm(vv);
+    }
   return 0;
 }
 
@@ -392,40 +461,59 @@ int oracle_van_pool(const double* van, int64_t n_slabs, int n_kv_heads, int64_t 
 // NULL). With van_pool != 0 the VaN stage ranks the layer-adaptive pooled
 // VaN (tau: the three CV thresholds; n_kv_heads groups slabs into layers;
 // src_fid goes with src_pid). pool_size_out: [n_slabs / n_kv_heads] or NULL.
+// With shared != 0 one index set per layer is chosen (scores of the
+// concatenated head blocks) and kept_out is [n_slabs / n_kv_heads][budget].
 int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
                     int64_t cap, int D, int64_t n_tokens, int p, int r,
                     int64_t budget, double alpha, const uint16_t* src_pid,
                     void* k_dst, void* v_dst, uint16_t* dst_pid, int32_t* kept_out,
                     int van_pool, const double* tau, int n_kv_heads, int grid_w,
-                    const uint32_t* src_fid, uint32_t* dst_fid, int32_t* pool_size_out) {
-  std::vector<double> tar(static_cast<size_t>(n_slabs * n_tokens));
+                    const uint32_t* src_fid, uint32_t* dst_fid, int32_t* pool_size_out,
+                    int shared) {
+  // With a shared index set the scores, the selection and kept_out are per
+  // layer ("units" = layers); else per slab.
+  if (n_kv_heads <= 0 || n_slabs % n_kv_heads != 0) return -1;
+  const int64_t H = shared ? n_kv_heads : 1;
+  const int64_t units = n_slabs / H;
+  std::vector<double> tar(static_cast<size_t>(units * n_tokens));
   std::vector<double> van(tar.size());
   if (n_tokens > budget) {
-    if (oracle_scores(k, v, is_bf16, n_slabs, cap, D, n_tokens, p, r, src_pid,
-                      tar.data(), van.data()) != 0)
-      return -1;
+    const int rc = shared ? oracle_scores_shared(k, v, is_bf16, units, static_cast<int>(H), cap, D,
+                                                 n_tokens, p, r, src_pid, tar.data(), van.data())
+                          : oracle_scores(k, v, is_bf16, n_slabs, cap, D, n_tokens, p, r, src_pid,
+                                          tar.data(), van.data());
+    if (rc != 0) return -1;
     if (van_pool) {
       if (grid_w <= 0 || p % grid_w != 0) return -1;
       std::vector<double> all(tar.size());
-      if (oracle_van_all(v, is_bf16, n_slabs, cap, D, n_tokens, all.data()) != 0) return -1;
-      if (oracle_van_pool(all.data(), n_slabs, n_kv_heads, n_tokens, p / grid_w, grid_w,
-                          src_pid, src_fid, cap, tau, van.data(), pool_size_out,
+      const int rv = shared ? oracle_van_all_shared(v, is_bf16, units, static_cast<int>(H), cap, D,
+                                                    n_tokens, all.data())
+                            : oracle_van_all(v, is_bf16, n_slabs, cap, D, n_tokens, all.data());
+      if (rv != 0) return -1;
+      // A layer is one unit of H heads, or (shared) one unit on its own; the
+      // ids of a shared unit are those of its first head.
+      if (oracle_van_pool(all.data(), units, shared ? 1 : n_kv_heads, n_tokens, p / grid_w,
+                          grid_w, src_pid, src_fid, cap * H, tau, van.data(), pool_size_out,
                           nullptr) != 0)
         return -1;
     }
   }
-  if (oracle_select(tar.data(), van.data(), n_slabs, n_tokens, p, r, budget, alpha,
-                    kept_out, nullptr) != 0)
+  int32_t* kept_sel = kept_out;
+  if (oracle_select(tar.data(), van.data(), units, n_tokens, p, r, budget, alpha,
+                    kept_sel, nullptr) != 0)
     return -1;
   if (n_tokens <= budget) return 0;  // pass-through leaves the cache as it is
+  // Every head of a unit is compacted with the unit's indices.
+  std::vector<int32_t> kept_slab(static_cast<size_t>(n_slabs * budget));
+  for (int64_t s = 0; s < n_slabs; ++s)
+    for (int64_t j = 0; j < budget; ++j) kept_slab[s * budget + j] = kept_sel[(s / H) * budget + j];
+  const int32_t* kept = kept_slab.data();
   const int64_t row_bytes = static_cast<int64_t>(D) * (is_bf16 ? 2 : 4);
-  if (oracle_gather_rows(k, k_dst, row_bytes, n_slabs, cap, cap, kept_out, budget) != 0) return -1;
-  if (oracle_gather_rows(v, v_dst, row_bytes, n_slabs, cap, cap, kept_out, budget) != 0) return -1;
-  if (dst_pid &&
-      oracle_gather_patch(src_pid, dst_pid, n_slabs, cap, cap, p, kept_out, budget) != 0)
+  if (oracle_gather_rows(k, k_dst, row_bytes, n_slabs, cap, cap, kept, budget) != 0) return -1;
+  if (oracle_gather_rows(v, v_dst, row_bytes, n_slabs, cap, cap, kept, budget) != 0) return -1;
+  if (dst_pid && oracle_gather_patch(src_pid, dst_pid, n_slabs, cap, cap, p, kept, budget) != 0)
     return -1;
-  if (dst_fid &&
-      oracle_gather_frame(src_fid, dst_fid, n_slabs, cap, cap, p, kept_out, budget) != 0)
+  if (dst_fid && oracle_gather_frame(src_fid, dst_fid, n_slabs, cap, cap, p, kept, budget) != 0)
     return -1;
   return 0;
 }

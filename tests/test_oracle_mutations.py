@@ -2,8 +2,8 @@
 
 Each case plants one mistake (a flipped sign, a dropped term, a wrong index,
 a wrong tie-break, ...) in a copy of oracle/ipv_oracle.cpp, builds the copy on
-the CPU, and runs the pin suites (test_oracle_pins.py, test_oracle_pool_pins.py)
-against it. Every
+the CPU, and runs the pin suites (test_oracle_pins.py, test_oracle_pool_pins.py,
+test_oracle_shared_pins.py) against it. Every
 mutant must make that suite fail; the unmutated copy must pass it.
 """
 import os
@@ -65,6 +65,14 @@ MUTANTS = [
      "if (oracle_van_pool(van.data(),"),
     ("selection ranks raw VaN", "tau, van.data(), pool_size_out,",
      "tau, all.data(), pool_size_out,"),
+    # per-layer shared index set
+    ("shared blocks hold only the first head", "  for (int h = 0; h < H; ++h) {\n    load_row(base, is_bf16, l * H + h, cap, D, n, row);",
+     "  for (int h = 0; h < 1; ++h) {\n    load_row(base, is_bf16, l * H + h, cap, D, n, row);"),
+    ("shared layer reads another layer's heads", "load_row(base, is_bf16, l * H + h, cap, D, n, row);",
+     "load_row(base, is_bf16, l + h, cap, D, n, row);"),
+    ("shared compaction uses the head's own index row",
+     "kept_slab[s * budget + j] = kept_sel[(s / H) * budget + j];",
+     "kept_slab[s * budget + j] = kept_sel[(s % H) * budget + j];"),
     ("frame ids of a fresh cache compacted as patch ids",
      "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n / p)",
      "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n % p)"),
@@ -75,7 +83,8 @@ def _run_pins_with(lib_path: str) -> int:
     env = dict(os.environ, IPV_ORACLE_LIB_OVERRIDE=lib_path)
     cmd = [sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
            os.path.join(ROOT, "tests", "test_oracle_pins.py"),
-           os.path.join(ROOT, "tests", "test_oracle_pool_pins.py")]
+           os.path.join(ROOT, "tests", "test_oracle_pool_pins.py"),
+           os.path.join(ROOT, "tests", "test_oracle_shared_pins.py")]
     return subprocess.run(cmd, env=env, cwd=ROOT, capture_output=True, timeout=300).returncode
 
 
@@ -97,6 +106,7 @@ def test_unmutated_copy_passes(tmp_path):
 def test_mutant_is_caught(tmp_path, name, old, new):
     with open(SRC) as fh:
         text = fh.read()
-    assert text.count(old) == 1, f"mutation anchor not unique/present: {old!r}"
+    # A line the per-head and the shared-head scoring share is mutated in both.
+    assert text.count(old) >= 1, f"mutation anchor not present: {old!r}"
     lib = _build_variant(tmp_path, "mutant", text.replace(old, new))
     assert _run_pins_with(lib) != 0, f"pins did not catch: {name}"
