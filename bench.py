@@ -27,7 +27,7 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "compress-pass latency (ms) and HBM GB/s vs GB300 peak, 7B shape 6K budget"
-KERNELS = ("recent_mean", "score", "select", "gather", "pipeline", "pool")
+KERNELS = ("recent_mean", "score", "select", "gather", "pipeline", "pool", "combine")
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -37,6 +37,8 @@ def workload_desc(w: synth.Workload) -> str:
          f"{w.n_frames} frames ({w.n_tokens} tokens) -> budget {w.budget}, alpha {w.tar_ratio}")
     if w.van_pool:
         d += f", layer-adaptive pooled VaN (CV thresholds {tuple(w.cv_tau)})"
+    if w.head_shared:
+        d += ", one index set per layer shared by its KV heads"
     return d
 
 
@@ -64,12 +66,23 @@ def bytes_model(w: synth.Workload, S: int, r: int):
         "gather": S * (4 * C * row + 4 * C),
         "pipeline": pass_bytes,  # the single-kernel pass does all four steps
         "pool": 0,
+        "combine": 0,
     }
     if w.van_pool:
         # the recent rows' V (and their VaN) for the layer's CV; the pooling
         # reads the VaN of every row and writes the pooled VaN of past rows
         per_kernel["recent_mean"] += S * (rp * row + 4 * rp)
         per_kernel["pool"] = S * (4 * N + 4 * n_past)
+    if w.head_shared:
+        # partial sums (k.m, |k|^2, |v|^2) of every head in, the layer's TaR and
+        # VaN out; the selection reads per-layer scores and writes per-layer kept
+        L = S // w.n_kv_heads
+        per_kernel["combine"] = S * 12 * n_past + L * 8 * n_past
+        per_kernel["score"] += S * 4 * n_past
+        per_kernel["select"] = L * (8 * n_past + 4 * C)
+        per_kernel["gather"] = S * 4 * C * row + L * 4 * C
+        if w.van_pool:
+            per_kernel["pool"] = L * (4 * N + 4 * n_past)
     return pass_bytes, tight, per_kernel
 
 
@@ -77,6 +90,10 @@ def oracle_pass(w: synth.Workload, k_np, v_np, r: int):
     """One oracle pass over the given slabs (pooled VaN if the workload asks
     for it; then the slabs are whole layers)."""
     import oracle
+    if w.head_shared:
+        return oracle.compress_shared(k_np, v_np, w.n_tokens, w.grid_h, w.grid_w, r, w.budget,
+                                      w.tar_ratio, w.n_kv_heads,
+                                      tau=w.cv_tau if w.van_pool else None)
     if w.van_pool:
         return oracle.compress_pooled(k_np, v_np, w.n_tokens, w.grid_h, w.grid_w, r, w.budget,
                                       w.tar_ratio, w.cv_tau, w.n_kv_heads)
@@ -173,7 +190,7 @@ def time_oracle(w: synth.Workload, k_np, v_np, r: int, budget_s: float = 12.0):
     import oracle
     oracle.build()
     S_total = w.n_slabs
-    unit = w.n_kv_heads if w.van_pool else 1  # pooled VaN needs whole layers
+    unit = w.n_kv_heads if (w.van_pool or w.head_shared) else 1  # whole layers
     t0 = time.perf_counter()
     oracle_pass(w, k_np[:unit], v_np[:unit], r)
     t1 = (time.perf_counter() - t0) / unit
@@ -194,7 +211,7 @@ def run_reference(args, w: synth.Workload):
     import oracle
     oracle.build()
     r = oracle.recent_frames(w.n_frames)
-    unit = w.n_kv_heads if w.van_pool else 1  # pooled VaN needs whole layers
+    unit = w.n_kv_heads if (w.van_pool or w.head_shared) else 1  # whole layers
     K1, V1 = synth.host_generate(w.scaled(n_streams=1), slabs=unit)
     t0 = time.perf_counter()
     oracle_pass(w, K1, V1, r)
@@ -233,7 +250,7 @@ def run_e2e(args, w, cache, kept, flush, one_pass, S, N, C, D):
     v_host = torch.empty_like(k_host, pin_memory=True)
     k_host.copy_(cache.k[0])
     v_host.copy_(cache.v[0])
-    kept_host = torch.empty((S, C), dtype=torch.int32, pin_memory=True)
+    kept_host = torch.empty(tuple(kept.shape), dtype=torch.int32, pin_memory=True)
     k_out = torch.empty((S, C, D), dtype=cache.k.dtype, pin_memory=True)
     v_out = torch.empty_like(k_out, pin_memory=True)
 
@@ -284,9 +301,10 @@ def run_stream(args, w: synth.Workload):
     S, N, C, D, p = w.slabs_per_stream, w.n_tokens, w.budget, w.head_dim, w.p
     ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
              token_capacity=N, single_kernel=args.single_kernel, van_pool=w.van_pool,
-             cv_tau=w.cv_tau)
+             cv_tau=w.cv_tau, head_shared=w.head_shared)
     r = ipv.recent_frames(w.n_frames)
-    kept = torch.empty((S, C), dtype=torch.int32, device="cuda")
+    kept = torch.empty((S // w.n_kv_heads if w.head_shared else S, C), dtype=torch.int32,
+                       device="cuda")
     pid_block = torch.arange(w.append_frames * p, device="cuda").remainder(p).to(torch.int16)
 
     def stream(timed: bool, profile_passes: int = 0):
@@ -426,13 +444,14 @@ def run_gpu(args, w: synth.Workload):
 
     ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
              token_capacity=N, single_kernel=args.single_kernel, van_pool=w.van_pool,
-             cv_tau=w.cv_tau)
+             cv_tau=w.cv_tau, head_shared=w.head_shared)
     r = ipv.recent_frames(w.n_frames)
     cache = PingPongCache(S, N, D, w.dtype, patch_ids=False)
     for i, st in enumerate(streams):
         synth.device_generate(w, cache.k[0, i * per:(i + 1) * per], cache.v[0, i * per:(i + 1) * per],
                               stream=st)
-    kept = torch.empty((S, C), dtype=torch.int32, device="cuda")
+    kept = torch.empty((S // w.n_kv_heads if w.head_shared else S, C), dtype=torch.int32,
+                       device="cuda")
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
     L = len(streams) * w.n_layers
 

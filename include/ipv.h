@@ -95,6 +95,15 @@ typedef struct {
                              g(CV) = 7 if CV < tau_1, 5 if CV < tau_2, 3 if
                              CV < tau_3, else 1 (Algorithm 2; the paper's values
                              are model-specific and unpublished) */
+  int head_shared;        /* 0: one index set per (layer, KV head) slab;
+                             1: one per layer, shared by its KV heads (Sec. 3.1:
+                             K in R^{H x N x D} compressed as K[:, I, :]): a
+                             token's key and value are its H x D blocks, TaR
+                             uses their l2-normalised (Frobenius) cosine and
+                             VaN their norm, kept_idx_out is [n_layers][budget]
+                             and every head is compacted with its layer's
+                             indices. Needs single_kernel = 0 and
+                             n_kv_heads*head_dim*element size <= 2048 bytes. */
 } ipv_options;
 
 /* One tensor (K or V) of the ping-pong cache: two halves of identical
@@ -137,7 +146,8 @@ void ipv_shutdown(void);
  *   budget        : |C|, rows kept per slab; r*p < budget.
  *   tar_ratio     : alpha in [0, 1]; the TaR share is floor(alpha * budget).
  *   kept_idx_out  : device int32 [n_layers*n_kv_heads][budget]: the kept
- *                   source rows, ascending per slab.
+ *                   source rows, ascending per slab ([n_layers][budget],
+ *                   per layer, with head_shared).
  *   stream        : a cudaStream_t (NULL = legacy default stream).
  * Pass-through: if n_tokens <= budget nothing is evicted: kept_idx_out gets
  * 0..n_tokens-1 then -1 padding, no row is copied and cur is not flipped.
@@ -154,7 +164,8 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
 
 /* Steps (i) and (ii) only, for inspection and parity checks: fp32 s_TaR and
  * s_VaN of every token of every slab into tar_out / van_out (device,
- * [n_slabs][n_tokens]). Entries of the r recent frames are written as 0,
+ * [n_slabs][n_tokens]; [n_layers][n_tokens] of per-layer scores with
+ * head_shared). Entries of the r recent frames are written as 0,
  * except that with van_pool van_out holds the VaN of recent rows too (the
  * layer's CV counts every cached token). Requires n_tokens > r*p. Same
  * argument rules as ipv_compress (budget and tar_ratio aside); the caches are
@@ -208,8 +219,9 @@ const char* ipv_status_string(ipv_status s);
 /* Kernel timing for benchmarks: while enabled, ipv_compress and ipv_score
  * record CUDA events around each kernel on the call's stream. Kernel ids:
  * 0 recent-frame mean, 1 scoring, 2 selection, 3 compaction, 4 the
- * single-kernel pass, 5 VaN pooling. */
-#define IPV_NUM_KERNELS 6
+ * single-kernel pass, 5 VaN pooling, 6 the per-layer combination of head
+ * sums (head_shared). */
+#define IPV_NUM_KERNELS 7
 ipv_status ipv_profile_enable(int on);
 
 /* Waits (at most timeout_ms) for the recorded events, then writes per kernel

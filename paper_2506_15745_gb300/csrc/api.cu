@@ -27,6 +27,9 @@ struct State {
   float* van = nullptr;
   float* m = nullptr;     // [max_slabs][max_frame_tokens][max_head_dim]
   float* pooled = nullptr;  // [max_slabs][token_capacity], van_pool only
+  float* kk = nullptr;      // [max_slabs][token_capacity], head_shared only: per-head |k|^2
+  float* tar_l = nullptr;   // [max_slabs][token_capacity], head_shared only: per-layer scores
+  float* van_l = nullptr;
   ipv::PipeState* pstate = nullptr;
   unsigned* pflags = nullptr;  // [kPipeFlags][max_slabs]
   bool pipe_dirty = false;     // a failed launch may have left queue state behind
@@ -187,6 +190,59 @@ ipv_status after_launch(cudaError_t e, const char* what) {
   return e == cudaSuccess ? IPV_OK : cuda_fail(e, what);
 }
 
+// The shared index set reads a token's n_kv_heads head-rows as one block
+// (at most 128 16-byte chunks per lane group of the recent-frame mean).
+ipv_status check_shared(int n_kv_heads, int head_dim) {
+  if (static_cast<int64_t>(n_kv_heads) * head_dim * elem_bytes() > 2048)
+    return fail(IPV_EINVAL, "head_shared needs n_kv_heads*head_dim*element size <= 2048 bytes");
+  return IPV_OK;
+}
+
+// Steps (i)-(ii) with one index set per layer: the recent-frame mean of each
+// layer's head blocks, the heads' partial sums, and their combination into
+// per-layer TaR and VaN ([L][n_tokens] in tar_out, van_out).
+cudaError_t launch_shared_scores(const ipv::ScoreArgs& phys, int n_kv_heads, float* tar_out,
+                                 float* van_out, int zero_recent, cudaStream_t st) {
+  ipv::ScoreArgs am = phys;  // the layer view of the recent-frame mean
+  am.n_slabs = phys.n_slabs / n_kv_heads;
+  am.hs = n_kv_heads;
+  am.tar = tar_out;
+  am.van = van_out;
+  am.zero_recent = zero_recent;
+  am.van_recent = g.opt.van_pool;
+  am.kk = nullptr;
+  ipv::ScoreArgs a = phys;   // per head-slab partial sums into scratch
+  a.tar = g.tar;
+  a.van = g.van;
+  a.kk = g.kk;
+  a.zero_recent = 0;
+  a.van_recent = 0;
+  a.hs = 1;
+  prof_begin(0, st);
+  cudaError_t e = ipv::launch_recent_mean(am, st);
+  prof_end(0, st);
+  if (e != cudaSuccess) return e;
+  prof_begin(1, st);
+  e = ipv::launch_score(a, st);
+  prof_end(1, st);
+  if (e != cudaSuccess) return e;
+  ipv::CombineArgs c{};
+  c.dot = g.tar;
+  c.kk = g.kk;
+  c.vv = g.van;
+  c.tar = tar_out;
+  c.van = van_out;
+  c.n_layers = am.n_slabs;
+  c.n_tokens = phys.n_tokens;
+  c.n_past = phys.n_tokens - static_cast<int64_t>(phys.r) * phys.p;
+  c.hs = n_kv_heads;
+  c.num_sms = g.num_sms;
+  prof_begin(6, st);
+  e = ipv::launch_combine(c, st);
+  prof_end(6, st);
+  return e;
+}
+
 }  // namespace
 
 namespace ipv {
@@ -219,6 +275,9 @@ void ipv_shutdown(void) {
   cudaFree(g.van);
   cudaFree(g.m);
   cudaFree(g.pooled);
+  cudaFree(g.kk);
+  cudaFree(g.tar_l);
+  cudaFree(g.van_l);
   cudaFree(g.pstate);
   cudaFree(g.pflags);
   g = State{};
@@ -238,6 +297,9 @@ ipv_status ipv_init(const ipv_options* opt) {
   if (opt->single_kernel != 0 && opt->single_kernel != 1)
     return fail(IPV_EINVAL, "single_kernel must be 0 or 1");
   if (opt->van_pool != 0 && opt->van_pool != 1) return fail(IPV_EINVAL, "van_pool must be 0 or 1");
+  if (opt->head_shared != 0 && opt->head_shared != 1) return fail(IPV_EINVAL, "head_shared must be 0 or 1");
+  if (opt->head_shared && opt->single_kernel)
+    return fail(IPV_EINVAL, "head_shared runs with the step kernels only (single_kernel = 0)");
   if (opt->van_pool) {
     if (opt->single_kernel) return fail(IPV_EINVAL, "van_pool runs with the step kernels only (single_kernel = 0)");
     if (opt->max_frame_tokens > IPV_MAX_POOL_FRAME_TOKENS)
@@ -270,6 +332,9 @@ ipv_status ipv_init(const ipv_options* opt) {
   if (cudaMalloc(&s.tar, score_bytes) != cudaSuccess || cudaMalloc(&s.van, score_bytes) != cudaSuccess ||
       cudaMalloc(&s.m, m_bytes) != cudaSuccess ||
       (opt->van_pool && cudaMalloc(&s.pooled, score_bytes) != cudaSuccess) ||
+      (opt->head_shared && (cudaMalloc(&s.kk, score_bytes) != cudaSuccess ||
+                            cudaMalloc(&s.tar_l, score_bytes) != cudaSuccess ||
+                            cudaMalloc(&s.van_l, score_bytes) != cudaSuccess)) ||
       cudaMalloc(&s.pstate, sizeof(ipv::PipeState)) != cudaSuccess ||
       cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess) {
     cudaGetLastError();
@@ -277,10 +342,13 @@ ipv_status ipv_init(const ipv_options* opt) {
     cudaFree(s.van);
     cudaFree(s.m);
     cudaFree(s.pooled);
+    cudaFree(s.kk);
+    cudaFree(s.tar_l);
+    cudaFree(s.van_l);
     cudaFree(s.pstate);
     cudaFree(s.pflags);
     return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated",
-                (opt->van_pool ? 3 : 2) * score_bytes + m_bytes);
+                (2 + opt->van_pool + 3 * opt->head_shared) * score_bytes + m_bytes);
   }
   if ((e = cudaMemset(s.pstate, 0, sizeof(ipv::PipeState))) != cudaSuccess ||
       (e = cudaMemset(s.pflags, 0, flag_bytes)) != cudaSuccess) {
@@ -288,6 +356,9 @@ ipv_status ipv_init(const ipv_options* opt) {
     cudaFree(s.van);
     cudaFree(s.m);
     cudaFree(s.pooled);
+    cudaFree(s.kk);
+    cudaFree(s.tar_l);
+    cudaFree(s.van_l);
     cudaFree(s.pstate);
     cudaFree(s.pflags);
     return cuda_fail(e, "clearing the pipeline state");
@@ -335,6 +406,10 @@ ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_he
   a.van_recent = g.opt.van_pool;
   a.num_sms = g.num_sms;
   a.error = &g.pstate->error;
+  if (g.opt.head_shared) {  // per-layer scores [n_layers][n_tokens]
+    if ((s = check_shared(n_kv_heads, head_dim)) != IPV_OK) return s;
+    return after_launch(launch_shared_scores(a, n_kv_heads, tar_out, van_out, 1, st), "scoring kernels");
+  }
   prof_begin(0, st);
   cudaError_t e = ipv::launch_recent_mean(a, st);
   prof_end(0, st);
@@ -394,8 +469,10 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
                 static_cast<long long>(g.opt.token_capacity));
   cudaSetDevice(g.opt.device);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int64_t units = g.opt.head_shared ? n_layers : sh.S;  // rows of kept_idx_out
+  if (g.opt.head_shared && (s = check_shared(n_kv_heads, head_dim)) != IPV_OK) return s;
   if (n_tokens <= budget)
-    return after_launch(ipv::launch_passthrough(kept_idx_out, sh.S, n_tokens, budget, st),
+    return after_launch(ipv::launch_passthrough(kept_idx_out, units, n_tokens, budget, st),
                         "pass-through kernel");
   if (n_tokens > IPV_MAX_TOKENS)
     return fail(IPV_EINVAL, "n_tokens %lld exceeds IPV_MAX_TOKENS", static_cast<long long>(n_tokens));
@@ -427,9 +504,10 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   a.error = &g.pstate->error;
 
   ipv::SelectArgs sa{};
-  sa.tar = g.tar;
-  sa.van = g.opt.van_pool ? g.pooled : g.van;
-  sa.n_slabs = sh.S;
+  sa.tar = g.opt.head_shared ? g.tar_l : g.tar;
+  sa.van = g.opt.van_pool ? g.pooled : g.opt.head_shared ? g.van_l : g.van;
+  sa.n_slabs = units;
+  sa.pf_heads = g.opt.head_shared ? n_kv_heads : 1;
   sa.n_tokens = sh.N;
   sa.rp = sh.rp;
   sa.budget = budget;
@@ -452,6 +530,7 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   ga.row_bytes = sh.D * elem_bytes();
   ga.p = sh.p;
   ga.num_sms = g.num_sms;
+  ga.heads_per_kept = g.opt.head_shared ? n_kv_heads : 1;
 
   cudaError_t e;
   if (g.opt.single_kernel) {
@@ -500,25 +579,33 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   sa.v_pf = a.v;
   sa.cap_pf = g.opt.token_capacity;
   sa.row_bytes_pf = static_cast<int>(row_bytes);
-  prof_begin(0, st);
-  e = ipv::launch_recent_mean(a, st);
-  prof_end(0, st);
-  if (e != cudaSuccess) return cuda_fail(e, "recent-frame mean kernel");
-  prof_begin(1, st);
-  e = ipv::launch_score(a, st);
-  prof_end(1, st);
-  if (e != cudaSuccess) return cuda_fail(e, "scoring kernel");
+  if (g.opt.head_shared) {
+    e = launch_shared_scores(a, n_kv_heads, g.tar_l, g.van_l, 0, st);
+    if (e != cudaSuccess) return cuda_fail(e, "scoring kernels");
+  } else {
+    prof_begin(0, st);
+    e = ipv::launch_recent_mean(a, st);
+    prof_end(0, st);
+    if (e != cudaSuccess) return cuda_fail(e, "recent-frame mean kernel");
+    prof_begin(1, st);
+    e = ipv::launch_score(a, st);
+    prof_end(1, st);
+    if (e != cudaSuccess) return cuda_fail(e, "scoring kernel");
+  }
   if (g.opt.van_pool) {  // the VaN stage ranks layer-adaptive pooled VaN
+    // A layer is n_kv_heads slabs, or (shared index set) one unit whose ids
+    // are those of its first head.
+    const int hsh = g.opt.head_shared ? n_kv_heads : 1;
     ipv::PoolArgs pa{};
-    pa.van = g.van;
+    pa.van = g.opt.head_shared ? g.van_l : g.van;
     pa.pooled = g.pooled;
     pa.patch_id = k->patch_id[k->cur];
     pa.frame_id = pa.patch_id ? k->frame_id[k->cur] : nullptr;
-    pa.id_stride = g.opt.token_capacity;
-    pa.n_slabs = sh.S;
+    pa.id_stride = g.opt.token_capacity * hsh;
+    pa.n_slabs = units;
     pa.n_tokens = sh.N;
     pa.n_rows = sh.N - sh.rp;
-    pa.n_heads = n_kv_heads;
+    pa.n_heads = g.opt.head_shared ? 1 : n_kv_heads;
     pa.grid_h = frame_grid_h;
     pa.grid_w = frame_grid_w;
     for (int i = 0; i < 3; ++i) pa.tau[i] = g.opt.cv_tau[i];

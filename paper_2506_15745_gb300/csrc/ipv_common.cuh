@@ -169,6 +169,10 @@ struct ScoreArgs {
   float* van;
   int zero_recent;          // write 0 to the recent-frame entries of tar (and van unless van_recent)
   int van_recent;           // write the VaN of the recent rows to van (pooled VaN's CV counts them)
+  int hs;                   // recent-frame mean only: heads per token block (> 1: the shared index
+                            // set; slab s is layer s of hs heads, m is written per head-slab)
+  float* kk;                // scoring only: if set, write per-head partial sums instead of scores:
+                            // tar <- k.m_q, kk <- |k|^2, van <- |v|^2 (NaN without a patch)
   int num_sms;
   unsigned* error;          // device word: bit 2 set if a bulk-copy wait timed out
 };
@@ -197,6 +201,7 @@ struct SelectArgs {
   int64_t n_slabs, n_tokens;
   int64_t rp, n_tar, n_van, budget;
   int32_t* kept;      // [S][budget]
+  int pf_heads;       // head-slabs whose recent rows a block prefetches (0 or 1: its own)
 };
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
@@ -214,14 +219,29 @@ struct GatherArgs {
   uint16_t* pid_dst;        // nullptr: not written
   const uint32_t* fid_src;  // nullptr: frame = n div p
   uint32_t* fid_dst;        // nullptr: not written
-  const int32_t* kept;      // [S][budget]
+  const int32_t* kept;      // [S / heads_per_kept][budget]
   int64_t n_slabs, cap, budget;
   int row_bytes, p;
   int num_sms;
+  int heads_per_kept;       // head-slabs sharing one row of kept (0 or 1: one each)
 };
 
 int gather_cpl(int row_bytes);  // 16-byte chunks per lane of a half-warp row copy
 cudaError_t launch_gather(const GatherArgs& a, cudaStream_t st);
+
+// Shared index set: per-token TaR and VaN of a layer from its heads' partial
+// sums (combine.cu).
+struct CombineArgs {
+  const float* dot;  // [L*hs][n_tokens] per head-slab: k.m_q
+  const float* kk;   //                                |k|^2
+  const float* vv;   //                                |v|^2
+  float* tar;        // [L][n_tokens]: rows [0, n_past) written
+  float* van;
+  int64_t n_layers, n_tokens, n_past;
+  int hs;
+  int num_sms;
+};
+cudaError_t launch_combine(const CombineArgs& a, cudaStream_t st);
 
 // Layer-adaptive pooling of VaN (pool.cu): one block per slab.
 constexpr int kPoolThreads = 1024;

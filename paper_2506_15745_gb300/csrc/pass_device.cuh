@@ -23,7 +23,11 @@ __device__ __forceinline__ float group_sum(float x) {
 // the warp calls it). Sec. 3.1 Eq. (tar) regrouped:
 //   m_q = (1/r) sum_t' k_t' / max(|k_t'|, eps),  rows n_past + t' p + q.
 // col_ok false: the group has no column (it still joins the shuffles).
-template <typename T, int LPR, int CPL>
+// VIRT (the shared index set): s is a layer of a.hs heads and a token's key
+// is its hs head-rows read as one vector (Sec. 3.1, K in R^{H x N x D}): chunk
+// c of the group is chunk c mod cph of head c / cph, the norm runs over all
+// heads, and each head's part of m_q goes to that head-slab's table.
+template <typename T, int LPR, int CPL, bool VIRT = false>
 __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q, bool col_ok) {
   constexpr int P2 = Chunk<T>::kPairs;
   constexpr int E = Chunk<T>::kElems;
@@ -31,9 +35,21 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
   const int lane = threadIdx.x & 31;
   const int sub = lane % LPR;
   const int row_bytes = a.D * static_cast<int>(sizeof(T));
-  const int n_chunks = row_bytes / 16;
+  const int cph = row_bytes / 16;                 // chunks of one head-row
+  const int hs = VIRT ? a.hs : 1;
+  const int n_chunks = cph * hs;
   const int64_t n_past = a.n_tokens - static_cast<int64_t>(a.r) * a.p;
-  const char* kslab = static_cast<const char*>(a.k) + s * a.cap * row_bytes;
+  const int64_t slab0 = s * hs;                   // first head-slab of this token block
+  const char* kslab = static_cast<const char*>(a.k) + slab0 * a.cap * row_bytes;
+  int64_t coff[CPL];  // VIRT: byte offset of each chunk in a token block (else c * 16, inline)
+  if (VIRT) {
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) {
+      const int c = sub + LPR * i;
+      const int h = c / cph;
+      coff[i] = static_cast<int64_t>(h) * a.cap * row_bytes + (c - h * cph) * 16;
+    }
+  }
 
   float2 acc[CPL][P2];
 #pragma unroll
@@ -50,7 +66,7 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
 #pragma unroll
       for (int i = 0; i < CPL; ++i) {
         const int c = sub + LPR * i;
-        raw[b][i] = (ok && c < n_chunks) ? ld_stream(row + c * 16) : make_uint4(0, 0, 0, 0);
+        raw[b][i] = (ok && c < n_chunks) ? ld_stream(row + (VIRT ? coff[i] : c * 16)) : make_uint4(0, 0, 0, 0);
       }
     }
 #pragma unroll
@@ -74,7 +90,7 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
     }
   }
   if (a.van_recent) {  // VaN of the r recent rows of patch q (Sec. 3.2), for a layer's CV
-    const char* vslab = static_cast<const char*>(a.v) + s * a.cap * row_bytes;
+    const char* vslab = static_cast<const char*>(a.v) + slab0 * a.cap * row_bytes;
     for (int t0 = 0; t0 < a.r; t0 += kBatch) {  // uniform across the warp
       uint4 raw[kBatch][CPL];
 #pragma unroll
@@ -84,7 +100,7 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
 #pragma unroll
         for (int i = 0; i < CPL; ++i) {
           const int c = sub + LPR * i;
-          raw[b][i] = (ok && c < n_chunks) ? ld_stream(row + c * 16) : make_uint4(0, 0, 0, 0);
+          raw[b][i] = (ok && c < n_chunks) ? ld_stream(row + (VIRT ? coff[i] : c * 16)) : make_uint4(0, 0, 0, 0);
         }
       }
 #pragma unroll
@@ -105,14 +121,16 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
   }
   if (!col_ok) return;
   const float inv_r = 1.0f / static_cast<float>(a.r);
-  float* mrow = a.m + (s * a.p + q) * static_cast<int64_t>(a.D);
 #pragma unroll
   for (int i = 0; i < CPL; ++i) {
     const int c = sub + LPR * i;
     if (c < n_chunks) {
+      const int h = VIRT ? c / cph : 0;
+      const int cc = c - h * cph;
+      float* mrow = a.m + ((slab0 + h) * a.p + q) * static_cast<int64_t>(a.D);
 #pragma unroll
       for (int e = 0; e < P2; e += 2)
-        *reinterpret_cast<float4*>(mrow + c * E + 2 * e) =
+        *reinterpret_cast<float4*>(mrow + cc * E + 2 * e) =
             make_float4(acc[i][e].x * inv_r, acc[i][e].y * inv_r, acc[i][e + 1].x * inv_r,
                         acc[i][e + 1].y * inv_r);
     }
@@ -124,7 +142,6 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
       if (!a.van_recent) a.van[s * a.n_tokens + n] = 0.0f;
     }
   }
-
 }
 
 // Where score_segment reads the m table from.
@@ -220,8 +237,14 @@ __device__ __forceinline__ void score_segment(const ScoreArgs& a, int64_t s, int
         // max(|k|, eps) = sqrt(max(|k|^2, eps^2)). A patch id outside [0, p)
         // has no recent-frame partner: NaN scores rank below every number,
         // so such a token is never preferred.
-        tar[n] = q_ok ? -dot * rsqrtf(fmaxf(kk, kNormEps * kNormEps)) : __int_as_float(0x7fc00000);
-        van[n] = q_ok ? sqrtf(vv) : __int_as_float(0x7fc00000);
+        if (a.kk) {  // the shared index set: this head's partial sums
+          tar[n] = q_ok ? dot : __int_as_float(0x7fc00000);
+          a.kk[s * a.n_tokens + n] = kk;
+          van[n] = q_ok ? vv : __int_as_float(0x7fc00000);
+        } else {
+          tar[n] = q_ok ? -dot * rsqrtf(fmaxf(kk, kNormEps * kNormEps)) : __int_as_float(0x7fc00000);
+          van[n] = q_ok ? sqrtf(vv) : __int_as_float(0x7fc00000);
+        }
       }
     }
     q_base += step_mod;
@@ -865,7 +888,7 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
       if (t < g_end) {
         s = g / a.budget;
         j = g - s * a.budget;
-        n = a.kept[g];
+        n = a.heads_per_kept > 1 ? a.kept[(s / a.heads_per_kept) * a.budget + j] : a.kept[g];
         if (n >= a.cap) n = -1;  // never produced by the selection; ignore
       }
       src_n[u] = n;
@@ -918,10 +941,11 @@ __device__ __forceinline__ void gather_ids(const GatherArgs& a) {
   const int64_t total = a.n_slabs * a.budget;
   const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total; g += step) {
-    const int n = a.kept[g];
-    if (n < 0 || n >= a.cap) continue;
     const int64_t s = g / a.budget;
-    const int64_t dst = s * a.cap + (g - s * a.budget);
+    const int64_t j = g - s * a.budget;
+    const int n = a.heads_per_kept > 1 ? a.kept[(s / a.heads_per_kept) * a.budget + j] : a.kept[g];
+    if (n < 0 || n >= a.cap) continue;
+    const int64_t dst = s * a.cap + j;
     if (a.pid_dst)
       a.pid_dst[dst] = a.pid_src ? a.pid_src[s * a.cap + n] : static_cast<uint16_t>(n % a.p);
     if (a.fid_dst)

@@ -19,8 +19,9 @@ namespace {
 
 constexpr int kScoreThreads = 768;
 
-// m_q for 32/LPR patches per warp, patches flattened over (slab, q).
-template <typename T, int LPR, int CPL>
+// m_q for 32/LPR patches per warp, patches flattened over (slab, q); with
+// VIRT a "slab" is a layer whose a.hs heads form one token block.
+template <typename T, int LPR, int CPL, bool VIRT>
 __global__ void __launch_bounds__(128) recent_mean_kernel(ScoreArgs a) {
   pdl_trigger();
   constexpr int RPW = 32 / LPR;
@@ -30,7 +31,7 @@ __global__ void __launch_bounds__(128) recent_mean_kernel(ScoreArgs a) {
   const bool col_ok = col < a.n_slabs * a.p;
   const int64_t s = col_ok ? col / a.p : 0;
   const int q = col_ok ? static_cast<int>(col - s * a.p) : 0;
-  dev::mean_group<T, LPR, CPL>(a, s, q, col_ok);
+  dev::mean_group<T, LPR, CPL, VIRT>(a, s, q, col_ok);
 }
 
 // Streams the past rows. Block b owns an equal contiguous share of the
@@ -101,7 +102,11 @@ cudaError_t dispatch_score(const ScoreArgs& a, cudaStream_t st) {
 template <typename T, int LPR, int CPL>
 cudaError_t dispatch_mean(const ScoreArgs& a, cudaStream_t st) {
   const int64_t warps = (a.n_slabs * a.p + (32 / LPR) - 1) / (32 / LPR);
-  recent_mean_kernel<T, LPR, CPL><<<static_cast<unsigned>((warps * 32 + 127) / 128), 128, 0, st>>>(a);
+  const unsigned grid = static_cast<unsigned>((warps * 32 + 127) / 128);
+  if (a.hs > 1)
+    recent_mean_kernel<T, LPR, CPL, true><<<grid, 128, 0, st>>>(a);
+  else
+    recent_mean_kernel<T, LPR, CPL, false><<<grid, 128, 0, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -125,7 +130,9 @@ cudaError_t prepare_t() {
 
 template <typename T, bool MEAN>
 cudaError_t dispatch_t(const ScoreArgs& a, cudaStream_t st) {
-  switch (row_shape(a.D, a.is_bf16)) {
+  // The recent-frame mean of the shared index set reads hs head-rows per token.
+  const int width = MEAN && a.hs > 1 ? a.D * a.hs : a.D;
+  switch (row_shape(width, a.is_bf16)) {
     case 41: return MEAN ? dispatch_mean<T, 4, 1>(a, st) : dispatch_score<T, 4, 1>(a, st);
     case 42: return MEAN ? dispatch_mean<T, 4, 2>(a, st) : dispatch_score<T, 4, 2>(a, st);
     case 44: return MEAN ? dispatch_mean<T, 4, 4>(a, st) : dispatch_score<T, 4, 4>(a, st);

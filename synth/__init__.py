@@ -63,6 +63,7 @@ class Workload:
     value_locality: float = 0.0            # beta of the first layer (falls to 0 at the last)
     van_pool: bool = False                 # layer-adaptive VaN pooling in the pass
     cv_tau: tuple = (0.0, 0.0, 0.0)        # CV thresholds of the pool-size map
+    head_shared: bool = False              # one index set per layer for all its KV heads
 
     @property
     def p(self) -> int:
@@ -111,6 +112,9 @@ CONFIGS = {
     "llava_pool": Workload("llava_pool", 28, 4, 128, "bf16", 14, 14, 48, 6272, 0.5,
                            value_sigma=0.25, value_sigma_last=1.0, value_locality=0.9,
                            van_pool=True, cv_tau=(0.4, 0.6, 0.9)),
+    # the LLaVA shape with one index set per layer shared by its 4 KV heads
+    "llava_shared": Workload("llava_shared", 28, 4, 128, "bf16", 14, 14, 48, 6272, 0.5,
+                             head_shared=True),
     # the pooled workload streamed like "stream" (frame ids travel with the rows)
     "stream_pool": Workload("stream_pool", 28, 4, 128, "bf16", 14, 14, 48, 6272, 0.5,
                             value_sigma=0.25, value_sigma_last=1.0, value_locality=0.9,
