@@ -281,6 +281,74 @@ def run_e2e(args, w, cache, kept, flush, one_pass, S, N, C, D):
             "steps": e2e_steps}
 
 
+def steady_steps(w: synth.Workload, cache, S, C, D, p, rank, n_steps: int = 100):
+    """The stream's steady-state step (append the next frames behind the C
+    survivors with ipv_append_frames, then compress), launched eagerly and as
+    replays of two captured CUDA graphs (one per ping-pong parity). Host
+    submission time is taken while a sleep kernel holds the GPU, so it counts
+    only the enqueue cost; device time is events around all the steps."""
+    import torch
+
+    from paper_2506_15745_gb300 import ipv
+    if n_steps <= 0:
+        return None
+    gen = synth.DeviceGenerator(w, S, stream=rank)
+    nf = w.append_frames
+    k_new = torch.empty((S, nf * p, D), dtype=cache.k.dtype, device="cuda")
+    v_new = torch.empty_like(k_new)
+    gen.fill(k_new, v_new, 0, nf)
+    kept = torch.empty((S // w.n_kv_heads if w.head_shared else S, C), dtype=torch.int32, device="cuda")
+
+    def structs(c):
+        fids = (cache.fid[0], cache.fid[1]) if cache.fid is not None else (None, None)
+        k = ipv.KV.from_tensors((cache.k[0], cache.k[1]), (cache.pid[0], cache.pid[1]), c, fids)
+        v = ipv.KV.from_tensors((cache.v[0], cache.v[1]), (None, None), c)
+        return k, v
+
+    def step(c):
+        k, v = structs(c)
+        ipv.append_frames(k, v, k_new, v_new, w.n_layers, w.n_kv_heads, D, C, nf, w.grid_h, w.grid_w)
+        ipv.compress(k, v, w.n_layers, w.n_kv_heads, D, w.n_tokens, w.grid_h, w.grid_w, C,
+                     w.tar_ratio, kept)
+        return k.cur
+
+    torch.cuda.synchronize()
+    graphs = {}
+    for c in (0, 1):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            step(c)
+        graphs[c] = g
+    out = {"steps": n_steps, "appended_frames": nf}
+    for mode in ("eager", "graph"):
+        cur = cache.cur
+        for _ in range(3):  # warm-up
+            if mode == "graph":
+                graphs[cur].replay()
+                cur = 1 - cur
+            else:
+                cur = step(cur)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(200_000_000)  # ~0.1 s: the host enqueues every step meanwhile
+        e0.record()
+        t0 = time.perf_counter()
+        for _ in range(n_steps):
+            if mode == "graph":
+                graphs[cur].replay()
+                cur = 1 - cur
+            else:
+                cur = step(cur)
+        submit = time.perf_counter() - t0
+        e1.record()
+        torch.cuda.synchronize()
+        out[f"{mode}_submit_us_per_step"] = submit * 1e6 / n_steps
+        out[f"{mode}_device_ms_per_step"] = e0.elapsed_time(e1) / n_steps
+        cache.cur = cur
+    return out
+
+
 def run_stream(args, w: synth.Workload):
     """Streaming run (Algorithm 1 loop): frames are generated on the device and
     appended 16 at a time; whenever the cache holds n_tokens rows the pass
@@ -362,6 +430,7 @@ def run_stream(args, w: synth.Workload):
     p50 = max_over_ranks(float(np.percentile(per_pass, 50)))
     p99 = max_over_ranks(float(np.percentile(per_pass, 99)))
     total_ms = max_over_ranks(total_ms)
+    steady = steady_steps(w, cache, S, C, D, p, rank, n_steps=args.graph_steps) if world == 1 else None
 
     pass_bytes, tight_bytes, kbytes = bytes_model(w, S, r)
     peak, peak_kind = peaks()
@@ -409,6 +478,7 @@ def run_stream(args, w: synth.Workload):
             "gpu_launches": sum(prof[k][1] for k in KERNELS) * len(evs) // max(1, prof_passes),
             "timed_wall_s": t_wall,
             "clocks": clk,
+            "steady_step": steady,
         }
         print(json.dumps(line), flush=True)
     ipv.shutdown()
@@ -585,6 +655,8 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--config", default="llava", choices=sorted(synth.CONFIGS))
+    ap.add_argument("--graph-steps", type=int, default=100,
+                    help="streaming configs: steady-state steps timed eager and as CUDA-graph replays")
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--e2e-max-gb", type=float, default=8.0)

@@ -205,6 +205,29 @@ ipv_status ipv_van_pool(const float* van, const uint16_t* patch_id, const uint32
                         int frame_grid_h, int frame_grid_w, const float cv_tau[3],
                         float* pooled_out, int32_t* pool_size_out, void* stream);
 
+/* Algorithm 1's accumulate step ("accumulate KV embeddings until reaching
+ * |M|") for a streaming cache: appends n_new_frames whole frames behind the
+ * rows already cached, in every slab of the live halves buf[cur].
+ *   k_new, v_new : device [n_layers*n_kv_heads][n_new_frames*p][head_dim],
+ *                  contiguous, the element type of ipv_init (the model's K and
+ *                  V of the new frames, patch-major within a frame).
+ *   row0         : rows already cached per slab; the new rows go to row0 ..
+ *                  row0 + n_new_frames*p - 1 (row0 + those <= token_capacity).
+ *   Patch ids (if k->patch_id[cur]): the frame-grid position, (row - row0)
+ *   mod p. Frame ids (if k->frame_id[cur]): the frame id of row row0-1 plus
+ *   1, 2, ... per new frame, or first_frame, first_frame + 1, ... when row0
+ *   is 0; numbered on the device, so a captured CUDA graph that replays
+ *   "append, then ipv_compress" keeps counting frames. Together the two ids
+ *   are each row's position metadata: (frame, i, j) for a decoder that
+ *   re-applies rotary positions after compression (App. B.4), and the row
+ *   order for one that re-indexes positions 0..|M|-1.
+ * Enqueued on stream, no allocation, cur is not changed. Errors: IPV_EINVAL
+ * (NULL or misaligned pointers, non-positive sizes, rows beyond
+ * token_capacity, sizes above the ipv_init maxima), IPV_ENOINIT, IPV_ECUDA. */
+ipv_status ipv_append_frames(ipv_kv* k, ipv_kv* v, const void* k_new, const void* v_new, int n_layers,
+                             int n_kv_heads, int head_dim, int64_t row0, int n_new_frames,
+                             int frame_grid_h, int frame_grid_w, uint32_t first_frame, void* stream);
+
 /* The recent-frame count r the library uses for a cache of n_frames frames
  * (the ipv_init override if set, else max(1, floor(n_frames/8 + 1/2))).
  * Returns -1 before ipv_init. */

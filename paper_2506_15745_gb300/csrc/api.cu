@@ -673,6 +673,52 @@ ipv_status ipv_van_pool(const float* van, const uint16_t* patch_id, const uint32
   return after_launch(e, "VaN pooling kernel");
 }
 
+ipv_status ipv_append_frames(ipv_kv* k, ipv_kv* v, const void* k_new, const void* v_new, int n_layers,
+                             int n_kv_heads, int head_dim, int64_t row0, int n_new_frames,
+                             int frame_grid_h, int frame_grid_w, uint32_t first_frame, void* stream) {
+  if (!k || !v || !k_new || !v_new) return fail(IPV_EINVAL, "k, v, k_new and v_new must not be NULL");
+  if ((k->cur != 0 && k->cur != 1) || (v->cur != 0 && v->cur != 1)) return fail(IPV_EINVAL, "cur must be 0 or 1");
+  if (n_layers <= 0 || n_kv_heads <= 0 || head_dim <= 0 || n_new_frames <= 0 || frame_grid_h <= 0 ||
+      frame_grid_w <= 0 || row0 < 0)
+    return fail(IPV_EINVAL, "sizes must be positive and row0 >= 0");
+  const int64_t p = static_cast<int64_t>(frame_grid_h) * frame_grid_w;
+  if (p > 65535) return fail(IPV_EINVAL, "frame_grid_h*frame_grid_w exceeds 65535");
+  void* kd = k->buf[k->cur];
+  void* vd = v->buf[v->cur];
+  if (!kd || !vd || kd == vd) return fail(IPV_EINVAL, "live halves must be distinct and not NULL");
+  if (!aligned16(kd) || !aligned16(vd) || !aligned16(k_new) || !aligned16(v_new))
+    return fail(IPV_EINVAL, "cache halves and new rows must be 16-byte aligned");
+  const uint32_t* fid = k->frame_id[k->cur];
+  if (fid && (reinterpret_cast<uintptr_t>(fid) & 3u)) return fail(IPV_EINVAL, "frame ids must be 4-byte aligned");
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  const int64_t S = static_cast<int64_t>(n_layers) * n_kv_heads;
+  const int64_t n_new = static_cast<int64_t>(n_new_frames) * p;
+  if (S > g.opt.max_slabs) return fail(IPV_EINVAL, "n_layers*n_kv_heads exceeds max_slabs");
+  if (head_dim > g.opt.max_head_dim) return fail(IPV_EINVAL, "head_dim exceeds max_head_dim");
+  if ((static_cast<int64_t>(head_dim) * elem_bytes()) % 16 != 0)
+    return fail(IPV_EINVAL, "head_dim*element size must be a multiple of 16 bytes");
+  if (row0 + n_new > g.opt.token_capacity)
+    return fail(IPV_EINVAL, "row0 + %lld new rows exceed token_capacity %lld", static_cast<long long>(n_new),
+                static_cast<long long>(g.opt.token_capacity));
+  cudaSetDevice(g.opt.device);
+  ipv::AppendArgs a{};
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.k_dst = kd;
+  a.v_dst = vd;
+  a.pid = k->patch_id[k->cur];
+  a.fid = k->frame_id[k->cur];
+  a.n_slabs = S;
+  a.cap = g.opt.token_capacity;
+  a.row0 = row0;
+  a.n_new = n_new;
+  a.row_bytes = head_dim * elem_bytes();
+  a.p = static_cast<int>(p);
+  a.first_frame = first_frame;
+  a.num_sms = g.num_sms;
+  return after_launch(ipv::launch_append(a, static_cast<cudaStream_t>(stream)), "append kernel");
+}
+
 ipv_status ipv_device_error(uint32_t* err_out) {
   if (!err_out) return fail(IPV_EINVAL, "err_out must not be NULL");
   if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");

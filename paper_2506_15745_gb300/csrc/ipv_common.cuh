@@ -229,6 +229,21 @@ struct GatherArgs {
 int gather_cpl(int row_bytes);  // 16-byte chunks per lane of a half-warp row copy
 cudaError_t launch_gather(const GatherArgs& a, cudaStream_t st);
 
+// Appending whole frames to a streaming cache (append.cu).
+struct AppendArgs {
+  const void* k_new;   // [S][n_new][row_bytes], contiguous
+  const void* v_new;
+  void* k_dst;         // [S][cap][row_bytes]: rows row0 .. row0 + n_new - 1 written
+  void* v_dst;
+  uint16_t* pid;       // [S][cap] or nullptr
+  uint32_t* fid;       // [S][cap] or nullptr
+  int64_t n_slabs, cap, row0, n_new;
+  int row_bytes, p;
+  uint32_t first_frame;
+  int num_sms;
+};
+cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
+
 // Shared index set: per-token TaR and VaN of a layer from its heads' partial
 // sums (combine.cu).
 struct CombineArgs {

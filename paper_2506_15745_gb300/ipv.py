@@ -94,9 +94,11 @@ def load():
                                             I64, F, P, P]
         lib.ipv_van_pool.argtypes = [P, P, P, I64, I32, I32, I64, I32, I32,
                                      ctypes.POINTER(ctypes.c_float), P, P, P]
+        lib.ipv_append_frames.argtypes = [KVP, KVP, P, P, I32, I32, I32, I64, I32, I32, I32,
+                                          ctypes.c_uint32, P]
         for name in ("ipv_init", "ipv_compress", "ipv_score", "ipv_select",
                      "ipv_profile_enable", "ipv_profile_collect", "ipv_device_error",
-                     "ipv_compress_static", "ipv_van_pool"):
+                     "ipv_compress_static", "ipv_van_pool", "ipv_append_frames"):
             getattr(lib, name).restype = I32
         _lib = lib
     return _lib
@@ -186,6 +188,15 @@ def van_pool(van, n_layers: int, n_kv_heads: int, n_tokens: int, frame_grid_h: i
     _check(load().ipv_van_pool(_ptr(van), _ptr(patch_id), _ptr(frame_id), id_stride, n_layers,
                                n_kv_heads, n_tokens, frame_grid_h, frame_grid_w, tau,
                                _ptr(pooled_out), _ptr(pool_size_out), _stream(stream)))
+
+
+def append_frames(k: KV, v: KV, k_new, v_new, n_layers: int, n_kv_heads: int, head_dim: int,
+                  row0: int, n_new_frames: int, frame_grid_h: int, frame_grid_w: int,
+                  first_frame: int = 0, stream=None) -> None:
+    """ipv_append_frames: whole new frames behind row0 in every slab of the live halves."""
+    _check(load().ipv_append_frames(ctypes.byref(k), ctypes.byref(v), _ptr(k_new), _ptr(v_new),
+                                    n_layers, n_kv_heads, head_dim, row0, n_new_frames,
+                                    frame_grid_h, frame_grid_w, first_frame, _stream(stream)))
 
 
 def device_error() -> int:
