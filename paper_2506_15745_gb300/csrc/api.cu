@@ -507,7 +507,6 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   sa.tar = g.opt.head_shared ? g.tar_l : g.tar;
   sa.van = g.opt.van_pool ? g.pooled : g.opt.head_shared ? g.van_l : g.van;
   sa.n_slabs = units;
-  sa.pf_heads = g.opt.head_shared ? n_kv_heads : 1;
   sa.n_tokens = sh.N;
   sa.rp = sh.rp;
   sa.budget = budget;
@@ -531,6 +530,8 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   ga.p = sh.p;
   ga.num_sms = g.num_sms;
   ga.heads_per_kept = g.opt.head_shared ? n_kv_heads : 1;
+  ga.n_tokens = sh.N;
+  ga.rp = sh.rp;
 
   cudaError_t e;
   if (g.opt.single_kernel) {
@@ -571,14 +572,8 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
     return IPV_OK;
   }
 
-  // Overlap: while the (latency-bound) selection runs, it prefetches every
-  // slab's recent rows, which are always kept, into L2; the compaction copies
-  // them first (67 MB at the LLaVA shape, inside the 129 MB L2).
-  const int64_t row_bytes = static_cast<int64_t>(sh.D) * elem_bytes();
-  sa.k_pf = a.k;
-  sa.v_pf = a.v;
-  sa.cap_pf = g.opt.token_capacity;
-  sa.row_bytes_pf = static_cast<int>(row_bytes);
+  // Overlap: the compaction copies the recent rows (always kept) while the
+  // latency-bound selection runs (see gather.cu).
   if (g.opt.head_shared) {
     e = launch_shared_scores(a, n_kv_heads, g.tar_l, g.van_l, 0, st);
     if (e != cudaSuccess) return cuda_fail(e, "scoring kernels");

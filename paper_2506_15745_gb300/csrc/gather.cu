@@ -7,22 +7,28 @@
 //
 // Pure data movement (HBM-bound): a half-warp moves one 16-byte-chunked K row
 // and the matching V row; the flattened (slab, j) space is strided over the
-// whole grid with several rows in flight per half-warp. Patch and frame ids
-// travel with their rows, copied by a separate coalesced loop.
+// whole grid with several rows in flight per half-warp. The recent frames
+// (always kept, always the last rp kept rows) are copied before the kernel
+// waits for the selection, overlapping it. Patch and frame ids travel with
+// their rows, copied by a separate coalesced loop.
 #include "pass_device.cuh"
 
 namespace ipv {
 namespace {
 
 template <int CPL>
-__global__ void __launch_bounds__(512, 2) gather_kernel(GatherArgs a) {
+__global__ void __launch_bounds__(512, CPL >= 8 ? 1 : 2) gather_kernel(GatherArgs a) {
   pdl_trigger();
-  pdl_wait();  // the kept indices come from the selection kernel
   constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
   const int64_t n_hw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
   const int64_t hw = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 4;
+  // The recent frames are always kept, as the last rp kept rows: copy them
+  // while the selection is still running (it leaves HBM idle).
+  if (a.rp > 0) dev::gather_range<CPL, kU, false, false, true>(a, 0, a.n_slabs * a.rp, hw, n_hw, a.rp);
+  pdl_wait();  // the kept indices come from the selection kernel
   dev::gather_ids(a);
-  dev::gather_range<CPL, kU, true, false>(a, 0, a.n_slabs * a.budget, hw, n_hw);
+  const int64_t jn = a.budget - a.rp;  // the selected (past) rows of every slab
+  dev::gather_range<CPL, kU, false, false>(a, 0, a.n_slabs * jn, hw, n_hw, jn);
 }
 
 template <int CPL>

@@ -103,12 +103,6 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Asks the bulk-copy engine to bring [p, p + bytes) into L2 (no data is
-// returned; bytes a multiple of 16, p 16-byte aligned).
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
-
 // Bounded wait for a barrier phase; false if it did not complete in time.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   for (int it = 0; it < (1 << 22); ++it)
@@ -194,14 +188,9 @@ cudaError_t score_prepare(int max_p, int max_D);
 struct SelectArgs {
   const float* tar;   // [S][n_tokens]
   const float* van;
-  const void* k_pf;   // if set: K/V halves whose recent rows are prefetched into L2
-  const void* v_pf;   // for the compaction that follows ([S][cap][row_bytes])
-  int64_t cap_pf;
-  int row_bytes_pf;
   int64_t n_slabs, n_tokens;
   int64_t rp, n_tar, n_van, budget;
   int32_t* kept;      // [S][budget]
-  int pf_heads;       // head-slabs whose recent rows a block prefetches (0 or 1: its own)
 };
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
@@ -224,6 +213,8 @@ struct GatherArgs {
   int row_bytes, p;
   int num_sms;
   int heads_per_kept;       // head-slabs sharing one row of kept (0 or 1: one each)
+  int64_t n_tokens, rp;     // rp > 0: the last rp kept rows of every slab are the rows
+                            // n_tokens - rp .. n_tokens - 1 (the recent frames, always kept)
 };
 
 int gather_cpl(int row_bytes);  // 16-byte chunks per lane of a half-warp row copy

@@ -217,6 +217,8 @@ extern "C" ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype,
   ga.row_bytes = head_dim * elem;
   ga.p = static_cast<int>(p);
   ga.num_sms = dev->num_sms;
+  ga.n_tokens = n_tokens;
+  ga.rp = rp;
   if ((e = ipv::launch_gather(ga, cs)) != cudaSuccess) return cuda_reject(e, "compaction kernel");
   k->cur = 1 - k->cur;
   v->cur = 1 - v->cur;

@@ -863,9 +863,14 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
 // Kept indices and source patch ids are read with plain loads (the kept
 // indices may have been written earlier in the same kernel). IDS: copy the
 // patch and frame ids of each row here too (else gather_ids does it).
-template <int CPL, int kU, bool REVERSE = false, bool IDS = true>
+// JN > 0 (the step kernels): g runs over (slab, j) with j < jn kept rows per
+// slab, the kept stride staying a.budget; FIXED: the source row is
+// a.n_tokens - a.rp + j and kept is not read (the recent frames, j < rp,
+// written to rows budget - rp + j).
+template <int CPL, int kU, bool REVERSE = false, bool IDS = true, bool FIXED = false>
 __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begin, int64_t g_end,
-                                             int64_t hw, int64_t n_hw) {
+                                             int64_t hw, int64_t n_hw, int64_t jn = 0) {
+  const int64_t per = jn > 0 ? jn : a.budget;  // (slab, j) rows per slab in g
   const int lane = threadIdx.x & 15;
   const int n_chunks = a.row_bytes / 16;
   const char* ks = static_cast<const char*>(a.k_src);
@@ -886,9 +891,14 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
       int n = -1;
       int64_t s = 0, j = 0;
       if (t < g_end) {
-        s = g / a.budget;
-        j = g - s * a.budget;
-        n = a.heads_per_kept > 1 ? a.kept[(s / a.heads_per_kept) * a.budget + j] : a.kept[g];
+        s = g / per;
+        j = g - s * per;
+        if (FIXED) {
+          n = static_cast<int>(a.n_tokens - a.rp + j);
+          j += a.budget - a.rp;
+        } else {
+          n = a.kept[(a.heads_per_kept > 1 ? s / a.heads_per_kept : s) * a.budget + j];
+        }
         if (n >= a.cap) n = -1;  // never produced by the selection; ignore
       }
       src_n[u] = n;
@@ -913,21 +923,13 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
           st_stream(vd + dst_off[u] + ch * 16, vr[u][c]);
         }
       }
-      if (IDS && a.pid_dst && lane == 0) {
-        const int64_t t = g0 + u * n_hw;
-        const int64_t g = REVERSE ? g_end - 1 - (t - g_begin) : t;
-        const int64_t s = g / a.budget;
-        const int64_t j = g - s * a.budget;
-        a.pid_dst[s * a.cap + j] = a.pid_src ? a.pid_src[s * a.cap + src_n[u]]
-                                             : static_cast<uint16_t>(src_n[u] % a.p);
-      }
-      if (IDS && a.fid_dst && lane == 1) {  // frame ids travel with their rows too
-        const int64_t t = g0 + u * n_hw;
-        const int64_t g = REVERSE ? g_end - 1 - (t - g_begin) : t;
-        const int64_t s = g / a.budget;
-        const int64_t j = g - s * a.budget;
-        a.fid_dst[s * a.cap + j] = a.fid_src ? a.fid_src[s * a.cap + src_n[u]]
-                                             : static_cast<uint32_t>(src_n[u] / a.p);
+      if (IDS && (a.pid_dst || a.fid_dst) && lane < 2) {  // ids travel with their rows too
+        const int64_t drow = dst_off[u] / a.row_bytes;       // s * cap + j
+        const int64_t srow = drow - (drow % a.cap) + src_n[u];
+        if (lane == 0 && a.pid_dst)
+          a.pid_dst[drow] = a.pid_src ? a.pid_src[srow] : static_cast<uint16_t>(src_n[u] % a.p);
+        if (lane == 1 && a.fid_dst)
+          a.fid_dst[drow] = a.fid_src ? a.fid_src[srow] : static_cast<uint32_t>(src_n[u] / a.p);
       }
     }
   }

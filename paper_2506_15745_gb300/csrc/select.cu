@@ -10,16 +10,6 @@ __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a)
   extern __shared__ uint32_t sm_sel[];
   __shared__ dev::SelShared sh;
   pdl_trigger();
-  // The selection is latency-bound: meanwhile, start moving this slab's
-  // recent rows (always kept) into L2 for the compaction that follows.
-  const int pf = a.pf_heads > 1 ? a.pf_heads : 1;  // head-slabs sharing this block's indices
-  if (a.k_pf && threadIdx.x < 2 * pf) {
-    const int64_t n_past = a.n_tokens - a.rp;
-    const int64_t slab = static_cast<int64_t>(blockIdx.x) * pf + (threadIdx.x >> 1);
-    const char* base = static_cast<const char*>((threadIdx.x & 1) ? a.v_pf : a.k_pf);
-    prefetch_l2(base + (slab * a.cap_pf + n_past) * a.row_bytes_pf,
-                static_cast<uint32_t>(a.rp * a.row_bytes_pf));
-  }
   pdl_wait();  // the scores come from the scoring kernel
   dev::select_slab<kSelectThreads>(a, blockIdx.x, sm_sel, sh);
 }
