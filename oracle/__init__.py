@@ -67,7 +67,9 @@ def _load():
         lib.oracle_gather_patch.argtypes = [P, P, I64, I64, I64, I32, P, I64]
         lib.oracle_gather_patch.restype = I32
         lib.oracle_compress.argtypes = [P, P, I32, I64, I64, I32, I64, I32, I32, I64, D,
-                                        P, P, P, P, P, I32, P, I32, I32, P, P, P, I32]
+                                        P, P, P, P, P, I32, P, I32, I32, P, P, P, I32, I32]
+        lib.oracle_frame_mean.argtypes = [P, I64, I64, I64, I32, P, I64]
+        lib.oracle_frame_mean.restype = I32
         lib.oracle_scores_shared.argtypes = [P, P, I32, I64, I32, I64, I32, I64, I32, I32, P, P, P]
         lib.oracle_scores_shared.restype = I32
         lib.oracle_van_all_shared.argtypes = [P, I32, I64, I32, I64, I32, I64, P]
@@ -193,7 +195,7 @@ def compress(k: np.ndarray, v: np.ndarray, n_tokens: int, p: int, r: int, budget
         patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
     rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
                                  budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
-                                 _ptr(pd), _ptr(kept), 0, None, 1, 0, None, None, None, 0)
+                                 _ptr(pd), _ptr(kept), 0, None, 1, 0, None, None, None, 0, 0)
     if rc != 0:
         raise ValueError("oracle_compress rejected its arguments")
     return kept, kd, vd, pd
@@ -264,7 +266,7 @@ def compress_pooled(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, gr
     rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
                                  budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
                                  _ptr(pd), _ptr(kept), 1, _ptr(_tau(tau)), n_kv_heads,
-                                 grid_w, _ptr(frame_id), _ptr(fd), _ptr(ks), 0)
+                                 grid_w, _ptr(frame_id), _ptr(fd), _ptr(ks), 0, 0)
     if rc != 0:
         raise ValueError("oracle_compress rejected its arguments")
     return kept, kd, vd, pd, fd, ks
@@ -324,7 +326,48 @@ def compress_shared(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, gr
                                  budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
                                  _ptr(pd), _ptr(kept), int(pooled),
                                  _ptr(_tau(tau)) if pooled else None, n_kv_heads, grid_w,
-                                 _ptr(frame_id), _ptr(fd), _ptr(ks), 1)
+                                 _ptr(frame_id), _ptr(fd), _ptr(ks), 1, 0)
     if rc != 0:
         raise ValueError("oracle_compress rejected its arguments")
     return kept, kd, vd, pd, fd, ks
+
+
+ABLATIONS = {"tar_reverse": 1, "van_reverse": 2, "tar_frame": 3}
+
+
+def frame_mean(tar: np.ndarray, n_past: int, p: int, frame_id: np.ndarray | None = None) -> np.ndarray:
+    """Frame-level TaR: each past row's TaR replaced by its frame's mean (copy)."""
+    t = np.array(tar, dtype=np.float64, copy=True, order="C")
+    U, N = t.shape
+    stride = N
+    if frame_id is not None:
+        frame_id = np.ascontiguousarray(frame_id, dtype=np.uint32)
+        stride = frame_id.shape[1]
+    if _load().oracle_frame_mean(_ptr(t), U, N, n_past, p, _ptr(frame_id), stride) != 0:
+        raise ValueError("oracle_frame_mean rejected its arguments")
+    return t
+
+
+def compress_ablation(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, grid_w: int, r: int,
+                      budget: int, alpha: float, ablation: str, patch_id=None, frame_id=None):
+    """Whole per-head pass with an ablation variant ("tar_reverse", "van_reverse",
+    "tar_frame"). Returns (kept, K~, V~, patch ids, frame ids)."""
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    S, cap, D = k.shape
+    p = grid_h * grid_w
+    kd, vd = np.zeros_like(k), np.zeros_like(v)
+    pd = np.zeros((S, cap), np.uint16)
+    fd = np.zeros((S, cap), np.uint32)
+    kept = np.empty((S, budget), np.int32)
+    if patch_id is not None:
+        patch_id = np.ascontiguousarray(patch_id, dtype=np.uint16)
+    if frame_id is not None:
+        frame_id = np.ascontiguousarray(frame_id, dtype=np.uint32)
+    rc = _load().oracle_compress(_ptr(k), _ptr(v), _kv_kind(k), S, cap, D, n_tokens, p, r,
+                                 budget, float(alpha), _ptr(patch_id), _ptr(kd), _ptr(vd),
+                                 _ptr(pd), _ptr(kept), 0, None, 1, grid_w, _ptr(frame_id),
+                                 _ptr(fd), None, 0, ABLATIONS[ablation])
+    if rc != 0:
+        raise ValueError("oracle_compress rejected its arguments")
+    return kept, kd, vd, pd, fd

@@ -52,6 +52,12 @@
 // VaN is their Frobenius norm. Selection then runs once per layer and every
 // head of the layer is compacted with that layer's indices.
 //
+// Ablation variants (Sec. 4 ablation study, "TaR Reverse", "VaN Reverse",
+// "TaR Frame"), used when the pass is asked for one: a reversed stage keeps
+// the lowest scores instead of the highest (its scores negated; NaN still
+// ranks last, ties still go to the lower index); the frame-level TaR gives
+// each past token the mean TaR of the cached past tokens of its frame.
+//
 // Element types: bf16 (widened exactly: bits << 16) or fp32, widened to double.
 
 #include <algorithm>
@@ -456,6 +462,29 @@ int oracle_van_pool(const double* van, int64_t n_slabs, int n_kv_heads, int64_t 
   return 0;
 }
 
+// Frame-level TaR ("TaR Frame" ablation): every past row n of every unit
+// gets the mean of tar over the past rows of its frame (frame_id with
+// stride id_stride if given, else n div p). tar: [units][n_tokens], in place.
+int oracle_frame_mean(double* tar, int64_t units, int64_t n_tokens, int64_t n_past, int p,
+                      const uint32_t* frame_id, int64_t id_stride) {
+  if (!tar || p <= 0 || n_past < 0 || n_past > n_tokens) return -1;
+  for (int64_t u = 0; u < units; ++u) {
+    double* t = tar + u * n_tokens;
+    std::map<int64_t, std::pair<double, int64_t>> acc;  // frame -> (sum, count)
+    std::vector<int64_t> frame(n_past);
+    for (int64_t n = 0; n < n_past; ++n) {
+      frame[n] = frame_id ? static_cast<int64_t>(frame_id[u * id_stride + n]) : n / p;
+      acc[frame[n]].first += t[n];
+      acc[frame[n]].second += 1;
+    }
+    for (int64_t n = 0; n < n_past; ++n) {
+      const auto& a = acc[frame[n]];
+      t[n] = a.first / static_cast<double>(a.second);
+    }
+  }
+  return 0;
+}
+
 // One whole pass over slabs [0, n_slabs): scores, selection, compaction of K
 // and V (and of patch ids when dst_pid != NULL, of frame ids when dst_fid !=
 // NULL). With van_pool != 0 the VaN stage ranks the layer-adaptive pooled
@@ -463,13 +492,14 @@ int oracle_van_pool(const double* van, int64_t n_slabs, int n_kv_heads, int64_t 
 // src_fid goes with src_pid). pool_size_out: [n_slabs / n_kv_heads] or NULL.
 // With shared != 0 one index set per layer is chosen (scores of the
 // concatenated head blocks) and kept_out is [n_slabs / n_kv_heads][budget].
+// ablation: 0 none, 1 TaR Reverse, 2 VaN Reverse, 3 TaR Frame.
 int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
                     int64_t cap, int D, int64_t n_tokens, int p, int r,
                     int64_t budget, double alpha, const uint16_t* src_pid,
                     void* k_dst, void* v_dst, uint16_t* dst_pid, int32_t* kept_out,
                     int van_pool, const double* tau, int n_kv_heads, int grid_w,
                     const uint32_t* src_fid, uint32_t* dst_fid, int32_t* pool_size_out,
-                    int shared) {
+                    int shared, int ablation) {
   // With a shared index set the scores, the selection and kept_out are per
   // layer ("units" = layers); else per slab.
   if (n_kv_heads <= 0 || n_slabs % n_kv_heads != 0) return -1;
@@ -483,6 +513,12 @@ int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
                           : oracle_scores(k, v, is_bf16, n_slabs, cap, D, n_tokens, p, r, src_pid,
                                           tar.data(), van.data());
     if (rc != 0) return -1;
+    const int64_t n_past = n_tokens - static_cast<int64_t>(r) * p;
+    if (ablation == 3 && src_pid && !src_fid) return -1;  // frames need frame ids once compacted
+    if (ablation == 3 &&  // TaR Frame: a unit's ids are those of its first head
+        oracle_frame_mean(tar.data(), units, n_tokens, n_past, p, src_pid ? src_fid : nullptr,
+                          cap * H) != 0)
+      return -1;
     if (van_pool) {
       if (grid_w <= 0 || p % grid_w != 0) return -1;
       std::vector<double> all(tar.size());
@@ -499,6 +535,10 @@ int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
     }
   }
   int32_t* kept_sel = kept_out;
+  if (ablation == 1)  // TaR Reverse: the lowest TaR first
+    for (double& x : tar) x = -x;
+  if (ablation == 2)  // VaN Reverse: the lowest VaN first
+    for (double& x : van) x = -x;
   if (oracle_select(tar.data(), van.data(), units, n_tokens, p, r, budget, alpha,
                     kept_sel, nullptr) != 0)
     return -1;

@@ -3,7 +3,7 @@
 Each case plants one mistake (a flipped sign, a dropped term, a wrong index,
 a wrong tie-break, ...) in a copy of oracle/ipv_oracle.cpp, builds the copy on
 the CPU, and runs the pin suites (test_oracle_pins.py, test_oracle_pool_pins.py,
-test_oracle_shared_pins.py) against it. Every
+test_oracle_shared_pins.py, test_oracle_ablation_pins.py) against it. Every
 mutant must make that suite fail; the unmutated copy must pass it.
 """
 import os
@@ -73,6 +73,14 @@ MUTANTS = [
     ("shared compaction uses the head's own index row",
      "kept_slab[s * budget + j] = kept_sel[(s / H) * budget + j];",
      "kept_slab[s * budget + j] = kept_sel[(s % H) * budget + j];"),
+    # ablation variants
+    ("TaR Reverse does not reverse", "for (double& x : tar) x = -x;", "for (double& x : tar) x = x;"),
+    ("VaN Reverse reverses TaR", "for (double& x : van) x = -x;", "for (double& x : tar) x = -x;"),
+    ("frame mean over the whole slab",
+     "frame[n] = frame_id ? static_cast<int64_t>(frame_id[u * id_stride + n]) : n / p;",
+     "frame[n] = frame_id ? static_cast<int64_t>(frame_id[u * id_stride + n]) : 0;"),
+    ("frame mean divides by the frame size p", "t[n] = a.first / static_cast<double>(a.second);",
+     "t[n] = a.first / static_cast<double>(p);"),
     ("frame ids of a fresh cache compacted as patch ids",
      "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n / p)",
      "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n % p)"),
@@ -84,7 +92,8 @@ def _run_pins_with(lib_path: str) -> int:
     cmd = [sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
            os.path.join(ROOT, "tests", "test_oracle_pins.py"),
            os.path.join(ROOT, "tests", "test_oracle_pool_pins.py"),
-           os.path.join(ROOT, "tests", "test_oracle_shared_pins.py")]
+           os.path.join(ROOT, "tests", "test_oracle_shared_pins.py"),
+           os.path.join(ROOT, "tests", "test_oracle_ablation_pins.py")]
     return subprocess.run(cmd, env=env, cwd=ROOT, capture_output=True, timeout=300).returncode
 
 
