@@ -104,7 +104,23 @@ typedef struct {
                              and every head is compacted with its layer's
                              indices. Needs single_kernel = 0 and
                              n_kv_heads*head_dim*element size <= 2048 bytes. */
+  int ablation;           /* IPV_ABLATION_*: a variant of the ablation study
+                             (Sec. 4, ablation table) for comparisons; needs
+                             single_kernel = 0 */
 } ipv_options;
+
+/* Ablation variants (Sec. 4 ablation table). TAR_REVERSE / VAN_REVERSE: the
+ * stage keeps the past tokens of lowest TaR / VaN instead of highest (NaN
+ * still ranks last, ties still go to the lower index). TAR_FRAME: frame-level
+ * redundancy, each past token's TaR replaced by the mean TaR of the cached
+ * past tokens of its frame (needs frame ids once the cache holds patch ids,
+ * and frame_grid_h*frame_grid_w <= IPV_MAX_POOL_FRAME_TOKENS). */
+enum {
+  IPV_ABLATION_NONE = 0,
+  IPV_ABLATION_TAR_REVERSE = 1,
+  IPV_ABLATION_VAN_REVERSE = 2,
+  IPV_ABLATION_TAR_FRAME = 3
+};
 
 /* One tensor (K or V) of the ping-pong cache: two halves of identical
  * layout; buf[cur] holds the live rows. patch_id[h] and frame_id[h] may be
@@ -165,7 +181,8 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
 /* Steps (i) and (ii) only, for inspection and parity checks: fp32 s_TaR and
  * s_VaN of every token of every slab into tar_out / van_out (device,
  * [n_slabs][n_tokens]; [n_layers][n_tokens] of per-layer scores with
- * head_shared). Entries of the r recent frames are written as 0,
+ * head_shared; with the TAR_FRAME ablation tar_out holds the frame means the
+ * selection ranks). Entries of the r recent frames are written as 0,
  * except that with van_pool van_out holds the VaN of recent rows too (the
  * layer's CV counts every cached token). Requires n_tokens > r*p. Same
  * argument rules as ipv_compress (budget and tar_ratio aside); the caches are
@@ -243,7 +260,8 @@ const char* ipv_status_string(ipv_status s);
  * record CUDA events around each kernel on the call's stream. Kernel ids:
  * 0 recent-frame mean, 1 scoring, 2 selection, 3 compaction, 4 the
  * single-kernel pass, 5 VaN pooling, 6 the per-layer combination of head
- * sums (head_shared). */
+ * sums (head_shared). The frame-level TaR kernel of the TAR_FRAME ablation
+ * is not timed. */
 #define IPV_NUM_KERNELS 7
 ipv_status ipv_profile_enable(int on);
 

@@ -190,6 +190,22 @@ ipv_status after_launch(cudaError_t e, const char* what) {
   return e == cudaSuccess ? IPV_OK : cuda_fail(e, what);
 }
 
+// The "TaR Frame" ablation: each past row of each unit (slab, or layer with
+// the shared index set, whose ids are its first head's) takes its frame's
+// mean TaR.
+cudaError_t launch_tar_frame(float* tar, const ipv_kv* k, int64_t units, int hsh, const Shape& sh,
+                             cudaStream_t st) {
+  ipv::FrameMeanArgs fa{};
+  fa.tar = tar;
+  fa.frame_id = k->patch_id[k->cur] ? k->frame_id[k->cur] : nullptr;
+  fa.id_stride = g.opt.token_capacity * hsh;
+  fa.units = units;
+  fa.n_tokens = sh.N;
+  fa.n_past = sh.N - sh.rp;
+  fa.p = sh.p;
+  return ipv::launch_frame_mean(fa, st);
+}
+
 // The shared index set reads a token's n_kv_heads head-rows as one block
 // (at most 128 16-byte chunks per lane group of the recent-frame mean).
 ipv_status check_shared(int n_kv_heads, int head_dim) {
@@ -300,6 +316,12 @@ ipv_status ipv_init(const ipv_options* opt) {
   if (opt->head_shared != 0 && opt->head_shared != 1) return fail(IPV_EINVAL, "head_shared must be 0 or 1");
   if (opt->head_shared && opt->single_kernel)
     return fail(IPV_EINVAL, "head_shared runs with the step kernels only (single_kernel = 0)");
+  if (opt->ablation < IPV_ABLATION_NONE || opt->ablation > IPV_ABLATION_TAR_FRAME)
+    return fail(IPV_EINVAL, "unknown ablation %d", opt->ablation);
+  if (opt->ablation != IPV_ABLATION_NONE && opt->single_kernel)
+    return fail(IPV_EINVAL, "ablation variants run with the step kernels only (single_kernel = 0)");
+  if (opt->ablation == IPV_ABLATION_TAR_FRAME && opt->max_frame_tokens > IPV_MAX_POOL_FRAME_TOKENS)
+    return fail(IPV_EINVAL, "the frame-level TaR needs max_frame_tokens <= %d", IPV_MAX_POOL_FRAME_TOKENS);
   if (opt->van_pool) {
     if (opt->single_kernel) return fail(IPV_EINVAL, "van_pool runs with the step kernels only (single_kernel = 0)");
     if (opt->max_frame_tokens > IPV_MAX_POOL_FRAME_TOKENS)
@@ -406,9 +428,14 @@ ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_he
   a.van_recent = g.opt.van_pool;
   a.num_sms = g.num_sms;
   a.error = &g.pstate->error;
+  const bool tar_frame = g.opt.ablation == IPV_ABLATION_TAR_FRAME;
+  if (tar_frame && k->patch_id[k->cur] && !k->frame_id[k->cur])
+    return fail(IPV_EINVAL, "the frame-level TaR needs frame ids for a cache with patch ids");
   if (g.opt.head_shared) {  // per-layer scores [n_layers][n_tokens]
     if ((s = check_shared(n_kv_heads, head_dim)) != IPV_OK) return s;
-    return after_launch(launch_shared_scores(a, n_kv_heads, tar_out, van_out, 1, st), "scoring kernels");
+    cudaError_t e = launch_shared_scores(a, n_kv_heads, tar_out, van_out, 1, st);
+    if (e == cudaSuccess && tar_frame) e = launch_tar_frame(tar_out, k, n_layers, n_kv_heads, sh, st);
+    return after_launch(e, "scoring kernels");
   }
   prof_begin(0, st);
   cudaError_t e = ipv::launch_recent_mean(a, st);
@@ -417,6 +444,7 @@ ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_he
   prof_begin(1, st);
   e = ipv::launch_score(a, st);
   prof_end(1, st);
+  if (e == cudaSuccess && tar_frame) e = launch_tar_frame(tar_out, k, sh.S, 1, sh, st);
   return after_launch(e, "scoring kernel");
 }
 
@@ -483,6 +511,8 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
     return fail(IPV_EINVAL, "pooled VaN needs frame ids for a cache with patch ids");
   if (g.opt.van_pool && ipv::pool_smem_bytes(frame_grid_h, frame_grid_w, true) == 0)
     return fail(IPV_EINVAL, "frame too large for pooled VaN");
+  if (g.opt.ablation == IPV_ABLATION_TAR_FRAME && k->patch_id[k->cur] && !k->frame_id[k->cur])
+    return fail(IPV_EINVAL, "the frame-level TaR needs frame ids for a cache with patch ids");
 
   ipv::ScoreArgs a{};
   a.k = k->buf[k->cur];
@@ -507,6 +537,8 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   sa.tar = g.opt.head_shared ? g.tar_l : g.tar;
   sa.van = g.opt.van_pool ? g.pooled : g.opt.head_shared ? g.van_l : g.van;
   sa.n_slabs = units;
+  sa.neg_tar = g.opt.ablation == IPV_ABLATION_TAR_REVERSE;
+  sa.neg_van = g.opt.ablation == IPV_ABLATION_VAN_REVERSE;
   sa.n_tokens = sh.N;
   sa.rp = sh.rp;
   sa.budget = budget;
@@ -586,6 +618,11 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
     e = ipv::launch_score(a, st);
     prof_end(1, st);
     if (e != cudaSuccess) return cuda_fail(e, "scoring kernel");
+  }
+  if (g.opt.ablation == IPV_ABLATION_TAR_FRAME) {
+    e = launch_tar_frame(g.opt.head_shared ? g.tar_l : g.tar, k, units, g.opt.head_shared ? n_kv_heads : 1,
+                         sh, st);
+    if (e != cudaSuccess) return cuda_fail(e, "frame-level TaR kernel");
   }
   if (g.opt.van_pool) {  // the VaN stage ranks layer-adaptive pooled VaN
     // A layer is n_kv_heads slabs, or (shared index set) one unit whose ids

@@ -191,6 +191,7 @@ struct SelectArgs {
   int64_t n_slabs, n_tokens;
   int64_t rp, n_tar, n_van, budget;
   int32_t* kept;      // [S][budget]
+  int neg_tar, neg_van;  // ablation: the stage ranks its negated scores (the lowest first)
 };
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
@@ -264,6 +265,16 @@ struct PoolArgs {
   float tau[3];
 };
 size_t pool_smem_bytes(int grid_h, int grid_w, bool staged);  // 0 if a frame does not fit
+
+// Frame-level TaR ablation: each past row's score becomes its frame's mean.
+struct FrameMeanArgs {
+  float* tar;                // [units][n_tokens], rows [0, n_past) rewritten in place
+  const uint32_t* frame_id;  // [units][id_stride] or nullptr (frame = n div p)
+  int64_t id_stride;
+  int64_t units, n_tokens, n_past;
+  int p;
+};
+cudaError_t launch_frame_mean(const FrameMeanArgs& a, cudaStream_t st);
 cudaError_t pool_prepare();
 cudaError_t launch_pool(const PoolArgs& a, cudaStream_t st, bool pdl);
 

@@ -805,7 +805,7 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
   // TaR stage over all past tokens.
   Stats st{INFINITY, -INFINITY, 0u};
   for (int i = threadIdx.x; i < n_past; i += NT) {
-    const float v = tar[i] + 0.0f;
+    const float v = (a.neg_tar ? -tar[i] : tar[i]) + 0.0f;  // NaN stays NaN, -0 becomes +0
     key[i] = score_key(v);
     stats_add(st, v);
   }
@@ -825,7 +825,7 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
       if (pk.pick(key[i])) {
         key[i] = kExcluded;
       } else {
-        const float v = vb[b] + 0.0f;
+        const float v = (a.neg_van ? -vb[b] : vb[b]) + 0.0f;
         key[i] = score_key(v);
         stats_add(sv, v);
       }

@@ -414,7 +414,71 @@ __global__ void __launch_bounds__(kPoolThreads, 1) pool_kernel(PoolArgs pa) {
   else pool_staged<1>(pa, ids, sv, out, n_rows, L, maps, ij, s_van, s_fid, s_pid);
 }
 
+// Frame-level TaR (the "TaR Frame" ablation): every past row of unit
+// blockIdx.x takes the mean of its frame's past-row scores. The rows of a
+// tile are staged in shared memory (score, frame id); each warp takes the
+// frames that start in its share, sums a frame lane by lane in row order then
+// across lanes (fixed order), and writes the mean to all its rows.
+constexpr int kMeanTile = 8192;
+
+__global__ void __launch_bounds__(1024, 1) frame_mean_kernel(FrameMeanArgs a) {
+  extern __shared__ float sm_fm[];
+  pdl_trigger();
+  pdl_wait();  // the scores come from the scoring kernels
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  float* t = a.tar + blockIdx.x * a.n_tokens;
+  const uint32_t* fid = a.frame_id ? a.frame_id + blockIdx.x * a.id_stride : nullptr;
+  const int n_past = static_cast<int>(a.n_past), p = a.p;
+  float* s_val = sm_fm;
+  uint32_t* s_fid = reinterpret_cast<uint32_t*>(sm_fm + kMeanTile + p + 1);
+  for (int t0 = 0; t0 < n_past; t0 += kMeanTile) {  // block-uniform
+    const int t1 = min(n_past, t0 + kMeanTile);
+    const int st0 = max(0, t0 - 1);
+    const int e1 = min(n_past, t1 + p);  // a frame is at most p rows
+    __syncthreads();
+    for (int m = st0 + threadIdx.x; m < e1; m += blockDim.x) {
+      s_val[m - st0] = t[m];
+      s_fid[m - st0] = fid ? fid[m] : static_cast<uint32_t>(m / p);
+    }
+    __syncthreads();
+    const int share = (t1 - t0 + nw - 1) / nw;
+    const int lo = t0 + warp * share, hi = min(t1, lo + share);
+    for (int base = lo; base < hi; base += 32) {  // warp-uniform
+      const int n = base + lane;
+      const bool st = n < hi && (n == 0 || s_fid[n - st0] != s_fid[n - 1 - st0]);
+      unsigned mask = __ballot_sync(0xffffffffu, st);
+      while (mask) {
+        const int f0 = base + __ffs(mask) - 1;
+        mask &= mask - 1;
+        const uint32_t f = s_fid[f0 - st0];
+        int f1 = e1;
+        for (int c = f0 + 1; c < e1; c += 32) {  // end of the run, inside the staging
+          const int mm = c + lane;
+          const unsigned other = __ballot_sync(0xffffffffu, mm < e1 && s_fid[mm - st0] != f);
+          if (other) {
+            f1 = c + __ffs(other) - 1;
+            break;
+          }
+        }
+        float sum = 0.0f;
+        for (int m = f0 + lane; m < f1; m += 32) sum += s_val[m - st0];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+        const float mean = sum / static_cast<float>(f1 - f0);
+        for (int m = f0 + lane; m < f1; m += 32) t[m] = mean;
+      }
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_frame_mean(const FrameMeanArgs& a, cudaStream_t st) {
+  if (a.p > kMaxPoolFrame) return cudaErrorInvalidValue;
+  const size_t smem = 2 * static_cast<size_t>(kMeanTile + a.p + 1) * sizeof(float);
+  cudaError_t e = launch(frame_mean_kernel, static_cast<unsigned>(a.units), 1024, smem, st, true, a);
+  return e == cudaSuccess ? cudaGetLastError() : e;
+}
 
 size_t pool_smem_bytes(int gh, int gw, bool staged) {
   const PoolLayout L = pool_layout(gh, gw);
@@ -426,8 +490,11 @@ size_t pool_smem_bytes(int gh, int gw, bool staged) {
 }
 
 cudaError_t pool_prepare() {
-  return cudaFuncSetAttribute(pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(kPoolSmem));
+  cudaError_t e = cudaFuncSetAttribute(pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(kPoolSmem));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(frame_mean_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(2 * (kMeanTile + kMaxPoolFrame + 1) * sizeof(float)));
 }
 
 cudaError_t launch_pool(const PoolArgs& a, cudaStream_t st, bool pdl) {
