@@ -305,6 +305,16 @@ ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype, int64_t to
  * since the last read) and clears it. Errors: IPV_ENOINIT, IPV_EINVAL, IPV_ECUDA. */
 ipv_status ipv_device_error(uint32_t* err_out);
 
+/* Diagnostic: the number of polls after which each wait of the single-kernel
+ * pass gives up (0 restores the default, 2^20 polls of about 0.1-0.3 us). A
+ * wait that gives up sets its bit in the device error word and the pass goes
+ * on without the awaited data: its results are then invalid, the device
+ * stays usable, and the next pass starts from a clean queue state. A short
+ * limit makes a pass fail fast instead of waiting; tests use it to exercise
+ * the error path. Takes effect at the next ipv_compress. Errors:
+ * IPV_EINVAL (negative), IPV_ENOINIT. */
+ipv_status ipv_set_wait_limit(int64_t polls);
+
 #ifdef __cplusplus
 }
 #endif

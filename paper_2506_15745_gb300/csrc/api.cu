@@ -33,6 +33,7 @@ struct State {
   ipv::PipeState* pstate = nullptr;
   unsigned* pflags = nullptr;  // [kPipeFlags][max_slabs]
   bool pipe_dirty = false;     // a failed launch may have left queue state behind
+  int64_t wait_limit = int64_t{1} << 20;  // polls before a wait of the single-kernel pass gives up
   bool profiling = false;
   std::vector<EventPair> pool;                      // idle event pairs
   std::vector<EventPair> pending[IPV_NUM_KERNELS];  // recorded, not yet read
@@ -587,7 +588,7 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
     pa.group = 4;
     pa.lead = 2;
     pa.n_groups = static_cast<int>((sh.S + pa.group - 1) / pa.group);
-    pa.spin_limit = int64_t{1} << 20;
+    pa.spin_limit = g.wait_limit;
     pa.nst = ipv::pipeline_stages(sh.p, sh.D, elem_bytes());
     // The selection needs its keys in shared memory as well (one item at a time).
     if (ipv::pipeline_smem_bytes(sh.N - sh.rp) > ipv::kBulkSmemMax)
@@ -749,6 +750,13 @@ ipv_status ipv_append_frames(ipv_kv* k, ipv_kv* v, const void* k_new, const void
   a.first_frame = first_frame;
   a.num_sms = g.num_sms;
   return after_launch(ipv::launch_append(a, static_cast<cudaStream_t>(stream)), "append kernel");
+}
+
+ipv_status ipv_set_wait_limit(int64_t polls) {
+  if (polls < 0) return fail(IPV_EINVAL, "polls must be >= 0");
+  if (!g.ready) return fail(IPV_ENOINIT, "ipv_init has not succeeded");
+  g.wait_limit = polls > 0 ? polls : int64_t{1} << 20;
+  return IPV_OK;
 }
 
 ipv_status ipv_device_error(uint32_t* err_out) {

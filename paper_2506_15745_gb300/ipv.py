@@ -95,11 +95,13 @@ def load():
                                             I64, F, P, P]
         lib.ipv_van_pool.argtypes = [P, P, P, I64, I32, I32, I64, I32, I32,
                                      ctypes.POINTER(ctypes.c_float), P, P, P]
+        lib.ipv_set_wait_limit.argtypes = [I64]
         lib.ipv_append_frames.argtypes = [KVP, KVP, P, P, I32, I32, I32, I64, I32, I32, I32,
                                           ctypes.c_uint32, P]
         for name in ("ipv_init", "ipv_compress", "ipv_score", "ipv_select",
                      "ipv_profile_enable", "ipv_profile_collect", "ipv_device_error",
-                     "ipv_compress_static", "ipv_van_pool", "ipv_append_frames"):
+                     "ipv_compress_static", "ipv_van_pool", "ipv_append_frames",
+                     "ipv_set_wait_limit"):
             getattr(lib, name).restype = I32
         _lib = lib
     return _lib
@@ -199,6 +201,11 @@ def append_frames(k: KV, v: KV, k_new, v_new, n_layers: int, n_kv_heads: int, he
     _check(load().ipv_append_frames(ctypes.byref(k), ctypes.byref(v), _ptr(k_new), _ptr(v_new),
                                     n_layers, n_kv_heads, head_dim, row0, n_new_frames,
                                     frame_grid_h, frame_grid_w, first_frame, _stream(stream)))
+
+
+def set_wait_limit(polls: int) -> None:
+    """ipv_set_wait_limit: polls before a single-kernel-pass wait gives up (0: default)."""
+    _check(load().ipv_set_wait_limit(int(polls)))
 
 
 def device_error() -> int:
