@@ -32,6 +32,7 @@ struct State {
   float* van_l = nullptr;
   ipv::PipeState* pstate = nullptr;
   unsigned* pflags = nullptr;  // [kPipeFlags][max_slabs]
+  unsigned* claim = nullptr;   // [2] compaction work counters, zero between passes
   bool pipe_dirty = false;     // a failed launch may have left queue state behind
   int64_t wait_limit = int64_t{1} << 20;  // polls before a wait of the single-kernel pass gives up
   bool profiling = false;
@@ -41,6 +42,14 @@ struct State {
 
 State g;
 thread_local std::string g_err;
+
+void free_scratch(State& s) {
+  for (void* p : {static_cast<void*>(s.tar), static_cast<void*>(s.van), static_cast<void*>(s.m),
+                  static_cast<void*>(s.pooled), static_cast<void*>(s.kk), static_cast<void*>(s.tar_l),
+                  static_cast<void*>(s.van_l), static_cast<void*>(s.pstate), static_cast<void*>(s.pflags),
+                  static_cast<void*>(s.claim)})
+    cudaFree(p);
+}
 
 ipv_status fail(ipv_status s, const char* fmt, ...) {
   char buf[512];
@@ -288,15 +297,7 @@ void ipv_shutdown(void) {
   cudaSetDevice(g.opt.device);
   cudaDeviceSynchronize();
   release_events();
-  cudaFree(g.tar);
-  cudaFree(g.van);
-  cudaFree(g.m);
-  cudaFree(g.pooled);
-  cudaFree(g.kk);
-  cudaFree(g.tar_l);
-  cudaFree(g.van_l);
-  cudaFree(g.pstate);
-  cudaFree(g.pflags);
+  free_scratch(g);
   g = State{};
 }
 
@@ -359,31 +360,16 @@ ipv_status ipv_init(const ipv_options* opt) {
                             cudaMalloc(&s.tar_l, score_bytes) != cudaSuccess ||
                             cudaMalloc(&s.van_l, score_bytes) != cudaSuccess)) ||
       cudaMalloc(&s.pstate, sizeof(ipv::PipeState)) != cudaSuccess ||
-      cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess) {
+      cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess || cudaMalloc(&s.claim, 2 * sizeof(unsigned)) != cudaSuccess) {
     cudaGetLastError();
-    cudaFree(s.tar);
-    cudaFree(s.van);
-    cudaFree(s.m);
-    cudaFree(s.pooled);
-    cudaFree(s.kk);
-    cudaFree(s.tar_l);
-    cudaFree(s.van_l);
-    cudaFree(s.pstate);
-    cudaFree(s.pflags);
+    free_scratch(s);
     return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated",
                 (2 + opt->van_pool + 3 * opt->head_shared) * score_bytes + m_bytes);
   }
   if ((e = cudaMemset(s.pstate, 0, sizeof(ipv::PipeState))) != cudaSuccess ||
-      (e = cudaMemset(s.pflags, 0, flag_bytes)) != cudaSuccess) {
-    cudaFree(s.tar);
-    cudaFree(s.van);
-    cudaFree(s.m);
-    cudaFree(s.pooled);
-    cudaFree(s.kk);
-    cudaFree(s.tar_l);
-    cudaFree(s.van_l);
-    cudaFree(s.pstate);
-    cudaFree(s.pflags);
+      (e = cudaMemset(s.pflags, 0, flag_bytes)) != cudaSuccess ||
+      (e = cudaMemset(s.claim, 0, 2 * sizeof(unsigned))) != cudaSuccess) {
+    free_scratch(s);
     return cuda_fail(e, "clearing the pipeline state");
   }
   s.ready = true;
@@ -565,6 +551,7 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   ga.heads_per_kept = g.opt.head_shared ? n_kv_heads : 1;
   ga.n_tokens = sh.N;
   ga.rp = sh.rp;
+  ga.claim = g.claim;
 
   cudaError_t e;
   if (g.opt.single_kernel) {

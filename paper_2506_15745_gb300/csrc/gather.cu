@@ -6,38 +6,72 @@
 // copy has no read/write hazards and the source stays intact.
 //
 // Pure data movement (HBM-bound): a half-warp moves one 16-byte-chunked K row
-// and the matching V row; the flattened (slab, j) space is strided over the
-// whole grid with several rows in flight per half-warp. The recent frames
-// (always kept, always the last rp kept rows) are copied before the kernel
-// waits for the selection, overlapping it. Patch and frame ids travel with
-// their rows, copied by a separate coalesced loop.
+// and the matching V row, several rows in flight per half-warp. The recent
+// frames (always kept, always the last rp kept rows) are copied before the
+// kernel waits for the selection, overlapping it: they are handed out in
+// chunks by a device counter, so the blocks that are already resident while
+// the selection runs (one beside each 1024-thread selection block, several on
+// the SMs it leaves free) copy all of them. The selected rows are then
+// strided over the whole grid. Patch and frame ids travel with their rows,
+// copied by a separate coalesced loop.
 #include "pass_device.cuh"
 
 namespace ipv {
 namespace {
 
+constexpr int kGatherThreads = 256;   // 64 registers: one block fits beside a selection block
+constexpr int64_t kRecentChunk = 128;  // recent rows per claim
+
 template <int CPL>
-__global__ void __launch_bounds__(512, CPL >= 8 ? 1 : 2) gather_kernel(GatherArgs a) {
+__global__ void __launch_bounds__(kGatherThreads, CPL >= 8 ? 2 : 4) gather_kernel(GatherArgs a) {
   pdl_trigger();
   constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
-  const int64_t n_hw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
-  const int64_t hw = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 4;
-  // The recent frames are always kept, as the last rp kept rows: copy them
-  // while the selection is still running (it leaves HBM idle).
-  if (a.rp > 0) dev::gather_range<CPL, kU, false, false, true>(a, 0, a.n_slabs * a.rp, hw, n_hw, a.rp);
+  if (a.rp > 0) {
+    __shared__ unsigned s_next;
+    const int64_t total = a.n_slabs * a.rp;
+    const int64_t n_chunks = (total + kRecentChunk - 1) / kRecentChunk;
+    if (threadIdx.x == 0) s_next = atomicAdd(a.claim, 1u);
+    __syncthreads();
+    unsigned c = s_next;
+    while (c < n_chunks) {  // block-uniform
+      unsigned nxt = 0;
+      if (threadIdx.x == 0) nxt = atomicAdd(a.claim, 1u);  // claimed ahead of need
+      const int64_t b0 = static_cast<int64_t>(c) * kRecentChunk;
+      dev::gather_range<CPL, kU, false, false, true>(a, b0, min(total, b0 + kRecentChunk), threadIdx.x >> 4,
+                                                     blockDim.x >> 4, a.rp);
+      __syncthreads();  // every thread has read s_next
+      if (threadIdx.x == 0) s_next = nxt;
+      __syncthreads();
+      c = s_next;
+    }
+  }
   pdl_wait();  // the kept indices come from the selection kernel
   dev::gather_ids(a);
+  const int64_t n_hw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
+  const int64_t hw = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 4;
   const int64_t jn = a.budget - a.rp;  // the selected (past) rows of every slab
   dev::gather_range<CPL, kU, false, false>(a, 0, a.n_slabs * jn, hw, n_hw, jn);
+  // The last block out clears the counters for the next pass. Every pass
+  // begins with a kernel launched without dependent-launch overlap, so the
+  // next compaction cannot start before this one has finished.
+  if (a.rp > 0 && threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(a.claim + 1, 1u) == gridDim.x - 1) {
+      a.claim[0] = 0;
+      a.claim[1] = 0;
+      __threadfence();
+    }
+  }
 }
 
 template <int CPL>
 cudaError_t dispatch(const GatherArgs& a, cudaStream_t st) {
   int per_sm = 0;
-  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gather_kernel<CPL>, 512, 0);
+  cudaError_t e =
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gather_kernel<CPL>, kGatherThreads, 0);
   if (e != cudaSuccess) return e;
   per_sm = per_sm < 1 ? 1 : per_sm;
-  return launch(gather_kernel<CPL>, a.num_sms * per_sm, 512, 0, st, true, a);
+  return launch(gather_kernel<CPL>, a.num_sms * per_sm, kGatherThreads, 0, st, true, a);
 }
 
 }  // namespace

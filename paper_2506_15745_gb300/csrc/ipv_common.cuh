@@ -216,6 +216,8 @@ struct GatherArgs {
   int heads_per_kept;       // head-slabs sharing one row of kept (0 or 1: one each)
   int64_t n_tokens, rp;     // rp > 0: the last rp kept rows of every slab are the rows
                             // n_tokens - rp .. n_tokens - 1 (the recent frames, always kept)
+  unsigned* claim;          // [2], zero between passes: recent-row chunks handed out, blocks
+                            // finished (the kernel clears both when it ends)
 };
 
 int gather_cpl(int row_bytes);  // 16-byte chunks per lane of a half-warp row copy

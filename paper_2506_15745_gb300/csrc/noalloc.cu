@@ -38,10 +38,13 @@ static_assert(IPV_STATIC_SCRATCH_BYTES % 256 == 0, "scratch size");
 
 // The working memory of every ipv_compress_static call on this device.
 static __device__ __align__(256) unsigned char g_static_scratch[IPV_STATIC_SCRATCH_BYTES];
+// The compaction's work counters (zero between passes).
+static __device__ unsigned g_static_claim[2];
 
 struct DeviceSetup {
   bool done = false;
   unsigned char* scratch = nullptr;  // device address of g_static_scratch
+  unsigned* claim = nullptr;         // device address of g_static_claim
   int num_sms = 0;
 };
 
@@ -78,6 +81,10 @@ ipv_status setup_current_device(DeviceSetup** out) {
     void* ptr = nullptr;
     if ((e = cudaGetSymbolAddress(&ptr, g_static_scratch)) != cudaSuccess)
       return cuda_reject(e, "cudaGetSymbolAddress of the static scratch");
+    void* cptr = nullptr;
+    if ((e = cudaGetSymbolAddress(&cptr, g_static_claim)) != cudaSuccess)
+      return cuda_reject(e, "cudaGetSymbolAddress of the compaction counters");
+    d.claim = static_cast<unsigned*>(cptr);
     if ((e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
       return cuda_reject(e, "cudaDeviceGetAttribute");
     d.scratch = static_cast<unsigned char*>(ptr);
@@ -219,6 +226,7 @@ extern "C" ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype,
   ga.num_sms = dev->num_sms;
   ga.n_tokens = n_tokens;
   ga.rp = rp;
+  ga.claim = dev->claim;
   if ((e = ipv::launch_gather(ga, cs)) != cudaSuccess) return cuda_reject(e, "compaction kernel");
   k->cur = 1 - k->cur;
   v->cur = 1 - v->cur;
