@@ -57,6 +57,9 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
 #pragma unroll
     for (int e = 0; e < P2; ++e) acc[i][e] = make_float2(0.0f, 0.0f);
 
+  // The recent K rows stay in L2 (evict-last) for the compaction, which
+  // copies them later in the pass; the scan in between is evict-first.
+  const uint64_t keep = l2_evict_last();
   for (int t0 = 0; t0 < a.r; t0 += kBatch) {  // uniform across the warp
     uint4 raw[kBatch][CPL];
 #pragma unroll
@@ -66,7 +69,8 @@ __device__ __forceinline__ void mean_group(const ScoreArgs& a, int64_t s, int q,
 #pragma unroll
       for (int i = 0; i < CPL; ++i) {
         const int c = sub + LPR * i;
-        raw[b][i] = (ok && c < n_chunks) ? ld_stream(row + (VIRT ? coff[i] : c * 16)) : make_uint4(0, 0, 0, 0);
+        raw[b][i] = (ok && c < n_chunks) ? ld_stream(row + (VIRT ? coff[i] : c * 16), keep)
+                                         : make_uint4(0, 0, 0, 0);
       }
     }
 #pragma unroll
@@ -184,6 +188,7 @@ __device__ __forceinline__ void score_segment(const ScoreArgs& a, int64_t s, int
   float* tar = a.tar + s * a.n_tokens;
   float* van = a.van + s * a.n_tokens;
   int q_base = lo % p;
+  const uint64_t once = l2_evict_first();  // read once: keep L2 for the recent rows
 
   for (int base = lo; base < hi; base += step) {
     uint4 kr[kU][CPL], vr[kU][CPL];
@@ -197,8 +202,8 @@ __device__ __forceinline__ void score_segment(const ScoreArgs& a, int64_t s, int
       for (int i = 0; i < CPL; ++i) {
         const int c = sub + LPR * i;
         const bool ld = ok && c < n_chunks;
-        kr[u][i] = ld ? ld_stream(kslab + ro + c * 16) : make_uint4(0, 0, 0, 0);
-        vr[u][i] = ld ? ld_stream(vslab + ro + c * 16) : make_uint4(0, 0, 0, 0);
+        kr[u][i] = ld ? ld_stream(kslab + ro + c * 16, once) : make_uint4(0, 0, 0, 0);
+        vr[u][i] = ld ? ld_stream(vslab + ro + c * 16, once) : make_uint4(0, 0, 0, 0);
       }
       int qi = q_base + off_mod[u];
       qi = qi >= p ? qi - p : qi;
@@ -842,14 +847,38 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
     if (pk.pick(key[i])) key[i] = kTaken;
   __syncthreads();
 
-  // Ascending kept indices: past picks, then the recent frames.
-  uint32_t mine = 0u;
-  for (int i = c0; i < c1; ++i) mine += (key[i] == kExcluded || key[i] == kTaken) ? 1u : 0u;
-  uint32_t total;
-  uint32_t pos = block_excl_scan<NT>(mine, &total, sh);
+  // Ascending kept indices: past picks, then the recent frames. Warp w
+  // compacts the picks of its own contiguous index range with ballots, so
+  // consecutive picks are stored by consecutive lanes.
+  constexpr int W = NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int span = ((n_past + W - 1) / W + 31) & ~31;  // indices per warp, a multiple of 32
+  const int w0 = min(n_past, warp * span), w1 = min(n_past, w0 + span);
+  uint32_t cnt = 0u;
+  for (int i0 = w0; i0 < w1; i0 += 32) {  // warp-uniform
+    const int i = i0 + lane;
+    cnt += __popc(__ballot_sync(0xffffffffu, i < w1 && (key[i] == kExcluded || key[i] == kTaken)));
+  }
+  if (lane == 0) sh.warp_a[warp] = cnt;
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t v = lane < W ? sh.warp_a[lane] : 0u;
+    const uint32_t incl = warp_incl_scan(v);
+    sh.warp_b[lane] = incl - v;
+    if (lane == 31) sh.bcast[7] = incl;
+  }
+  __syncthreads();
+  uint32_t pos = sh.warp_b[warp];
+  const uint32_t total = sh.bcast[7];
   int32_t* kept = a.kept + s * a.budget;
-  for (int i = c0; i < c1; ++i)
-    if ((key[i] == kExcluded || key[i] == kTaken) && pos < a.budget) kept[pos++] = i;
+  for (int i0 = w0; i0 < w1; i0 += 32) {
+    const int i = i0 + lane;
+    const bool pick = i < w1 && (key[i] == kExcluded || key[i] == kTaken);
+    const uint32_t m = __ballot_sync(0xffffffffu, pick);
+    const uint32_t at = pos + __popc(m & ((1u << lane) - 1u));
+    if (pick && at < a.budget) kept[at] = i;
+    pos += __popc(m);
+  }
   // total == n_tar + n_van by construction; the recent rows follow. The
   // guards only keep a broken count from writing outside this slab's row.
   for (int64_t j = threadIdx.x; j < a.rp; j += NT)
