@@ -32,7 +32,7 @@ struct State {
   float* van_l = nullptr;
   ipv::PipeState* pstate = nullptr;
   unsigned* pflags = nullptr;  // [kPipeFlags][max_slabs]
-  unsigned* claim = nullptr;   // [2] compaction work counters, zero between passes
+  unsigned* claim = nullptr;   // [3] compaction work counters, zero between passes
   bool pipe_dirty = false;     // a failed launch may have left queue state behind
   int64_t wait_limit = int64_t{1} << 20;  // polls before a wait of the single-kernel pass gives up
   bool profiling = false;
@@ -360,7 +360,7 @@ ipv_status ipv_init(const ipv_options* opt) {
                             cudaMalloc(&s.tar_l, score_bytes) != cudaSuccess ||
                             cudaMalloc(&s.van_l, score_bytes) != cudaSuccess)) ||
       cudaMalloc(&s.pstate, sizeof(ipv::PipeState)) != cudaSuccess ||
-      cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess || cudaMalloc(&s.claim, 2 * sizeof(unsigned)) != cudaSuccess) {
+      cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess || cudaMalloc(&s.claim, 3 * sizeof(unsigned)) != cudaSuccess) {
     cudaGetLastError();
     free_scratch(s);
     return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated",
@@ -368,7 +368,7 @@ ipv_status ipv_init(const ipv_options* opt) {
   }
   if ((e = cudaMemset(s.pstate, 0, sizeof(ipv::PipeState))) != cudaSuccess ||
       (e = cudaMemset(s.pflags, 0, flag_bytes)) != cudaSuccess ||
-      (e = cudaMemset(s.claim, 0, 2 * sizeof(unsigned))) != cudaSuccess) {
+      (e = cudaMemset(s.claim, 0, 3 * sizeof(unsigned))) != cudaSuccess) {
     free_scratch(s);
     return cuda_fail(e, "clearing the pipeline state");
   }

@@ -87,6 +87,14 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// 16-byte asynchronous copy from global into shared memory through L2 only
+// (cp.async.cg); a thread's copies complete at its cp_async_wait_all().
+// Both addresses are 16-byte aligned.
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
 }
@@ -239,8 +247,8 @@ struct GatherArgs {
   int heads_per_kept;       // head-slabs sharing one row of kept (0 or 1: one each)
   int64_t n_tokens, rp;     // rp > 0: the last rp kept rows of every slab are the rows
                             // n_tokens - rp .. n_tokens - 1 (the recent frames, always kept)
-  unsigned* claim;          // [2], zero between passes: recent-row chunks handed out, blocks
-                            // finished (the kernel clears both when it ends)
+  unsigned* claim;          // [3], zero between passes: recent-row and selected-row chunks
+                            // handed out, blocks finished (the kernel clears all three when it ends)
 };
 
 int gather_cpl(int row_bytes);  // 16-byte chunks per lane of a half-warp row copy

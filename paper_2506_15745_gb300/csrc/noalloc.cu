@@ -39,7 +39,7 @@ static_assert(IPV_STATIC_SCRATCH_BYTES % 256 == 0, "scratch size");
 // The working memory of every ipv_compress_static call on this device.
 static __device__ __align__(256) unsigned char g_static_scratch[IPV_STATIC_SCRATCH_BYTES];
 // The compaction's work counters (zero between passes).
-static __device__ unsigned g_static_claim[2];
+static __device__ unsigned g_static_claim[3];
 
 struct DeviceSetup {
   bool done = false;

@@ -58,12 +58,16 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(ScoreArgs a) {
     const float* m_slab = a.m + s * a.p * static_cast<int64_t>(a.D);
     if (SMEM_M) {
       __syncthreads();  // the previous slab's table is no longer read
+      // Every copy of the table is in flight at once: a row per warp and
+      // iteration with plain loads would take a dependent L2 round trip per
+      // row while the other SMs keep HBM saturated.
       const int d4 = a.D / 4;
       for (int q = warp; q < a.p; q += n_warps) {
         const float4* src = reinterpret_cast<const float4*>(m_slab + static_cast<int64_t>(q) * a.D);
         float4* dst = sm_m4 + q * (ms / 4);
-        for (int j = lane; j < d4; j += 32) dst[j] = __ldg(src + j);
+        for (int j = lane; j < d4; j += 32) cp_async16(dst + j, src + j);
       }
+      cp_async_wait_all();
       __syncthreads();
       dev::score_segment<T, LPR, CPL, kU, dev::kMSmem>(a, s, lo, hi,
                                                        reinterpret_cast<const float*>(sm_m4), ms);
