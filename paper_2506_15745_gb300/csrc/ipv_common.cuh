@@ -223,6 +223,7 @@ struct SelectArgs {
   int64_t rp, n_tar, n_van, budget;
   int32_t* kept;      // [S][budget]
   int neg_tar, neg_van;  // ablation: the stage ranks its negated scores (the lowest first)
+  int van_smem;       // set by launch_select: VaN is read into shared memory with TaR, up front
 };
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);

@@ -434,10 +434,11 @@ struct SelShared {
   uint32_t list_n;
 };
 
-// Shared memory of select_slab: keys[pad4(n_past)], hist[2048], list_key[NT], list_idx[NT].
+// Shared memory of select_slab: keys[pad4(n_past)], hist[2048], list_key[NT],
+// list_idx[NT], and with a.van_smem the VaN scores[pad4(n_past)].
 template <int NT>
-__host__ __device__ constexpr size_t select_smem_words(int64_t n_past) {
-  return static_cast<size_t>((n_past + 3) & ~3LL) + kSelectBins + 2 * NT;
+__host__ __device__ constexpr size_t select_smem_words(int64_t n_past, bool van_smem = false) {
+  return static_cast<size_t>((n_past + 3) & ~3LL) * (van_smem ? 2 : 1) + kSelectBins + 2 * NT;
 }
 
 __device__ __forceinline__ bool is_cand(uint32_t k) { return k != kExcluded && k != kTaken; }
@@ -718,15 +719,22 @@ __device__ Plan plan_stage(uint32_t* key, int n, uint32_t k, uint32_t n_cand, St
         }
         __syncthreads();
         const uint32_t m = min(sh.list_n, static_cast<uint32_t>(NT));
-        if (threadIdx.x < m) {
-          const uint32_t kt = list_key[threadIdx.x], it = list_idx[threadIdx.x];
-          uint32_t rank = 0u;
-          for (uint32_t j = 0; j < m; ++j) {
+        // T threads rank one candidate (T m <= NT, T <= 32, aligned within a
+        // warp), each against every T-th other one, then sum over the T lanes.
+        uint32_t T = 32u;
+        while (T > 1u && T * m > static_cast<uint32_t>(NT)) T >>= 1;
+        const uint32_t cand = threadIdx.x / T, sub = threadIdx.x % T;
+        uint32_t rank = 0u, kt = 0u, it = 0u;
+        if (cand < m) {
+          kt = list_key[cand];
+          it = list_idx[cand];
+          for (uint32_t j = sub; j < m; j += T) {
             const uint32_t kj = list_key[j];
             rank += (kj > kt || (kj == kt && list_idx[j] < it)) ? 1u : 0u;
           }
-          if (rank < k_rem) key[it] = mark;
         }
+        for (uint32_t off = T >> 1; off > 0u; off >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off);
+        if (cand < m && sub == 0u && rank < k_rem) key[it] = mark;
         __syncthreads();
         return P;
       }
@@ -807,10 +815,15 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
   const int c0 = min(n_past, static_cast<int>(threadIdx.x) * chunk);
   const int c1 = min(n_past, c0 + chunk);
 
+  // VaN goes to shared memory in the same pass as TaR when there is room,
+  // so that the VaN stage does not wait for a second round of loads.
+  float* vbuf = a.van_smem ? reinterpret_cast<float*>(list_idx + NT) : nullptr;
+
   // TaR stage over all past tokens.
   Stats st{INFINITY, -INFINITY, 0u};
   for (int i = threadIdx.x; i < n_past; i += NT) {
     const float v = (a.neg_tar ? -tar[i] : tar[i]) + 0.0f;  // NaN stays NaN, -0 becomes +0
+    if (vbuf) vbuf[i] = van[i];
     key[i] = score_key(v);
     stats_add(st, v);
   }
@@ -822,7 +835,7 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
   for (int i0 = c0; i0 < c1; i0 += 8) {
     float vb[8];  // issue the VaN loads of 8 tokens before using any
 #pragma unroll
-    for (int b = 0; b < 8; ++b) vb[b] = (i0 + b < c1) ? van[i0 + b] : 0.0f;
+    for (int b = 0; b < 8; ++b) vb[b] = (i0 + b < c1) ? (vbuf ? vbuf[i0 + b] : van[i0 + b]) : 0.0f;
 #pragma unroll
     for (int b = 0; b < 8; ++b) {
       const int i = i0 + b;

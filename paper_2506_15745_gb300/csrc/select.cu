@@ -30,14 +30,25 @@ size_t select_smem_bytes(int64_t n_past) {
   return dev::select_smem_words<kSelectThreads>(n_past) * sizeof(uint32_t);
 }
 
+namespace {
+// VaN in shared memory too while that stays within what select_prepare allows.
+bool van_fits(int64_t n_past) {
+  return dev::select_smem_words<kSelectThreads>(n_past, true) <=
+         dev::select_smem_words<kSelectThreads>(kMaxTokens);
+}
+}  // namespace
+
 cudaError_t select_prepare(int64_t max_tokens) {
   return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(select_smem_bytes(max_tokens)));
 }
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st) {
-  const size_t smem = select_smem_bytes(a.n_tokens - a.rp);
-  return launch(select_kernel, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st, true, a);
+  SelectArgs b = a;
+  const int64_t n_past = a.n_tokens - a.rp;
+  b.van_smem = van_fits(n_past) ? 1 : 0;
+  const size_t smem = dev::select_smem_words<kSelectThreads>(n_past, b.van_smem != 0) * sizeof(uint32_t);
+  return launch(select_kernel, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st, true, b);
 }
 
 cudaError_t launch_passthrough(int32_t* kept, int64_t n_slabs, int64_t n_tokens, int64_t budget,
