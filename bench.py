@@ -307,6 +307,19 @@ def run_e2e(args, w, cache, kept, flush, one_pass, S, N, C, D):
                     out_t[lo:hi].copy_(dev_t[1, lo:hi, :C], non_blocking=True)
                     drained[(lo, hi)][t] = d2h[t].record_event()
 
+    if small:  # latency-bound: the host's enqueue cost is the step, so keep it to six calls
+        k_all = ipv.KV.from_tensors((cache.k[0], cache.k[1]), (None, None), 0)
+        v_all = ipv.KV.from_tensors((cache.v[0], cache.v[1]), (None, None), 0)
+
+        def e2e_step():
+            cache.k[0].copy_(k_host, non_blocking=True)
+            cache.v[0].copy_(v_host, non_blocking=True)
+            k_all.cur = v_all.cur = 0
+            ipv.compress(k_all, v_all, n_layers, H, D, N, w.grid_h, w.grid_w, C, w.tar_ratio, kept, comp)
+            kept_host.copy_(kept, non_blocking=True)
+            k_out.copy_(cache.k[1, :, :C], non_blocking=True)
+            v_out.copy_(cache.v[1, :, :C], non_blocking=True)
+
     for _ in range(2):
         e2e_step()
     torch.cuda.synchronize()
