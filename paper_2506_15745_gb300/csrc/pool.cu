@@ -190,14 +190,21 @@ __host__ __device__ inline PoolLayout pool_layout(int gh, int gw) {
   return L;
 }
 
-// Pools every cached token of the frame rows [a, b) (a whole warp) directly:
-// the mean of the (VaN, 1) pairs in its (2 HALF + 1)^2 window of the
-// zero-padded map, read without bounds checks. The map is zero on entry and
-// on exit (the cells this frame set are cleared again). Rows come from the
-// block's staging: stage index m - st0.
+// Pools every cached token of the frame rows [a, b) (a whole warp): the mean
+// of the (VaN, 1) pairs in its (2 HALF + 1)^2 window of the zero-padded map.
+// The map is zero on entry and on exit. Rows come from the block's staging:
+// stage index m - st0. Two ways, whichever takes fewer shared-memory reads:
+//  - direct: every token sums its whole window, (2 HALF + 1)^2 reads each;
+//  - separable (p <= 32 kSepCells): each lane sums its interior cells along
+//    the grid row into registers, writes those row sums back over the map's
+//    interior, and every token then sums its column of row sums; padding
+//    rows and columns stay zero. All interior cells are cleared afterwards.
+constexpr int kSepCells = 8;  // interior cells per lane of the separable way
+
 template <int HALF>
 __device__ void pool_tokens(const PoolArgs& pa, int p, const float* s_van, const uint16_t* s_pid,
                             int st0, float* out, int a, int b, float2* map, const short2* ij) {
+  constexpr int W = 2 * HALF + 1;
   const int lane = threadIdx.x & 31;
   const int cp = pa.grid_w + 2 * kPad;
   for (int m = a + lane; m < b; m += 32) {
@@ -208,6 +215,38 @@ __device__ void pool_tokens(const PoolArgs& pa, int p, const float* s_van, const
     }
   }
   __syncwarp();
+  const int n = b - a;
+  const bool sep = p <= 32 * kSepCells && p * W + n * W + 2 * p < n * W * W;  // warp-uniform
+  if (sep) {
+    float2 rs[kSepCells];
+#pragma unroll
+    for (int u = 0; u < kSepCells; ++u) {
+      const int c = lane + 32 * u;
+      rs[u] = make_float2(0.0f, 0.0f);
+      if (c < p) {
+        const short2 t = ij[c];
+        const float2* r = map + (t.x + kPad) * cp + t.y + kPad;
+        float2 x[W];
+#pragma unroll
+        for (int dj = -HALF; dj <= HALF; ++dj) x[dj + HALF] = r[dj];
+#pragma unroll
+        for (int d = 0; d < W; ++d) {
+          rs[u].x += x[d].x;
+          rs[u].y += x[d].y;
+        }
+      }
+    }
+    __syncwarp();  // every row sum is read before any is written back
+#pragma unroll
+    for (int u = 0; u < kSepCells; ++u) {
+      const int c = lane + 32 * u;
+      if (c < p) {
+        const short2 t = ij[c];
+        map[(t.x + kPad) * cp + t.y + kPad] = rs[u];
+      }
+    }
+    __syncwarp();
+  }
   for (int m = a + lane; m < b; m += 32) {
     const int q = s_pid[m - st0];
     float y = __int_as_float(0x7fc00000);  // NaN: no grid position
@@ -215,16 +254,27 @@ __device__ void pool_tokens(const PoolArgs& pa, int p, const float* s_van, const
       const short2 t = ij[q];
       const float2* c = map + (t.x + kPad) * cp + t.y + kPad;
       float2 acc = make_float2(0.0f, 0.0f);
+      if (sep) {
+        float2 x[W];
 #pragma unroll
-      for (int di = -HALF; di <= HALF; ++di) {
-        const float2* r = c + di * cp;
-        float2 x[2 * HALF + 1];
+        for (int di = -HALF; di <= HALF; ++di) x[di + HALF] = c[di * cp];
 #pragma unroll
-        for (int dj = -HALF; dj <= HALF; ++dj) x[dj + HALF] = r[dj];
+        for (int d = 0; d < W; ++d) {
+          acc.x += x[d].x;
+          acc.y += x[d].y;
+        }
+      } else {
 #pragma unroll
-        for (int u = 0; u <= 2 * HALF; ++u) {
-          acc.x += x[u].x;
-          acc.y += x[u].y;
+        for (int di = -HALF; di <= HALF; ++di) {
+          const float2* r = c + di * cp;
+          float2 x[W];
+#pragma unroll
+          for (int dj = -HALF; dj <= HALF; ++dj) x[dj + HALF] = r[dj];
+#pragma unroll
+          for (int u = 0; u < W; ++u) {
+            acc.x += x[u].x;
+            acc.y += x[u].y;
+          }
         }
       }
       y = __fdividef(acc.x, acc.y);
@@ -232,11 +282,18 @@ __device__ void pool_tokens(const PoolArgs& pa, int p, const float* s_van, const
     out[m] = y;
   }
   __syncwarp();
-  for (int m = a + lane; m < b; m += 32) {
-    const int q = s_pid[m - st0];
-    if (q < p) {
-      const short2 t = ij[q];
+  if (sep) {
+    for (int c = lane; c < p; c += 32) {
+      const short2 t = ij[c];
       map[(t.x + kPad) * cp + t.y + kPad] = make_float2(0.0f, 0.0f);
+    }
+  } else {
+    for (int m = a + lane; m < b; m += 32) {
+      const int q = s_pid[m - st0];
+      if (q < p) {
+        const short2 t = ij[q];
+        map[(t.x + kPad) * cp + t.y + kPad] = make_float2(0.0f, 0.0f);
+      }
     }
   }
   __syncwarp();
@@ -263,11 +320,14 @@ __device__ void pool_staged(const PoolArgs& pa, const RowIds& ids, const float* 
     const int st0 = max(0, t0 - 1);                // one row before the tile: start detection
     const int e1 = min(n_rows, t1 + p);            // the tile's last frame ends before e1
     __syncthreads();                               // the previous tile's staging is no longer read
+    // The first tile's ids were staged before the wait for the scores.
 #pragma unroll 4
     for (int m = st0 + threadIdx.x; m < e1; m += blockDim.x) {
       s_van[m - st0] = sv[m];
-      s_fid[m - st0] = ids.fid[m];
-      s_pid[m - st0] = ids.pid[m];
+      if (t0 > 0) {
+        s_fid[m - st0] = ids.fid[m];
+        s_pid[m - st0] = ids.pid[m];
+      }
     }
     __syncthreads();
     if (warp >= L.nw) continue;
@@ -355,9 +415,35 @@ __global__ void __launch_bounds__(kPoolThreads, 1) pool_kernel(PoolArgs pa) {
   extern __shared__ float sm_pool[];
   __shared__ float2 red[33];
   pdl_trigger();
-  pdl_wait();  // VaN comes from the scoring kernels
   const int64_t s = blockIdx.x;
   const int64_t layer = s / pa.n_heads;
+
+  // What does not read the scores is set up before waiting for them: blocks
+  // that start on SMs the scoring kernel has already left do it meanwhile.
+  const int p = pa.grid_h * pa.grid_w;
+  const PoolLayout L = pool_layout(pa.grid_h, pa.grid_w);
+  float* maps = sm_pool;
+  short2* ij = reinterpret_cast<short2*>(maps + static_cast<size_t>(L.nw) * L.map_floats);
+  for (int c = threadIdx.x; c < p; c += blockDim.x)
+    ij[c] = make_short2(static_cast<short>(c / pa.grid_w), static_cast<short>(c % pa.grid_w));
+  RowIds ids;
+  ids.pid = pa.patch_id ? pa.patch_id + s * pa.id_stride : nullptr;
+  ids.fid = pa.frame_id ? pa.frame_id + s * pa.id_stride : nullptr;
+  ids.p = p;
+  const int n_rows = static_cast<int>(pa.n_rows);
+  float* s_van = reinterpret_cast<float*>(ij + p);
+  uint32_t* s_fid = reinterpret_cast<uint32_t*>(s_van + L.stage_rows);
+  uint16_t* s_pid = reinterpret_cast<uint16_t*>(s_fid + L.stage_rows);
+  if (ids.fid) {  // the zeroed maps and the first tile's ids (pool_staged's staging)
+    for (int i = threadIdx.x; i < L.nw * L.map_floats; i += blockDim.x) maps[i] = 0.0f;
+    const int e1 = min(n_rows, L.tile + p);
+#pragma unroll 4
+    for (int m = threadIdx.x; m < e1; m += blockDim.x) {
+      s_fid[m] = ids.fid[m];
+      s_pid[m] = ids.pid[m];
+    }
+  }
+  pdl_wait();  // VaN comes from the scoring kernels
 
   // Phase 1: CV of the layer (Algorithm 2: mu, sigma, CV = sigma / mu).
   const int64_t count = static_cast<int64_t>(pa.n_heads) * pa.n_tokens;
@@ -380,21 +466,9 @@ __global__ void __launch_bounds__(kPoolThreads, 1) pool_kernel(PoolArgs pa) {
     for (int64_t n = threadIdx.x; n < pa.n_rows; n += blockDim.x) out[n] = sv[n];
     return;
   }
-  const int p = pa.grid_h * pa.grid_w;
-  const PoolLayout L = pool_layout(pa.grid_h, pa.grid_w);
-  float* maps = sm_pool;
-  short2* ij = reinterpret_cast<short2*>(maps + static_cast<size_t>(L.nw) * L.map_floats);
-  for (int c = threadIdx.x; c < p; c += blockDim.x)
-    ij[c] = make_short2(static_cast<short>(c / pa.grid_w), static_cast<short>(c % pa.grid_w));
-  RowIds ids;
-  ids.pid = pa.patch_id ? pa.patch_id + s * pa.id_stride : nullptr;
-  ids.fid = pa.frame_id ? pa.frame_id + s * pa.id_stride : nullptr;
-  ids.p = p;
-  const int n_rows = static_cast<int>(pa.n_rows);
   const int warp = threadIdx.x >> 5;
   if (!ids.fid) {  // never compacted: whole p-row frames, dealt round-robin
-    __syncthreads();
-    if (warp >= L.nw) return;
+    if (warp >= L.nw) return;  // block_sum2's barriers published the (i, j) table
     float2* cell = reinterpret_cast<float2*>(maps + static_cast<size_t>(warp) * L.map_floats);
     float2* row = cell + p;
     for (int a = warp * p; a < n_rows; a += L.nw * p) {
@@ -405,10 +479,6 @@ __global__ void __launch_bounds__(kPoolThreads, 1) pool_kernel(PoolArgs pa) {
     }
     return;
   }
-  for (int i = threadIdx.x; i < L.nw * L.map_floats; i += blockDim.x) maps[i] = 0.0f;
-  float* s_van = reinterpret_cast<float*>(ij + p);
-  uint32_t* s_fid = reinterpret_cast<uint32_t*>(s_van + L.stage_rows);
-  uint16_t* s_pid = reinterpret_cast<uint16_t*>(s_fid + L.stage_rows);
   if (k == 7) pool_staged<3>(pa, ids, sv, out, n_rows, L, maps, ij, s_van, s_fid, s_pid);
   else if (k == 5) pool_staged<2>(pa, ids, sv, out, n_rows, L, maps, ij, s_van, s_fid, s_pid);
   else pool_staged<1>(pa, ids, sv, out, n_rows, L, maps, ij, s_van, s_fid, s_pid);
