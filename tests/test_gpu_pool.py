@@ -168,6 +168,36 @@ def test_van_pool_compacted_many_tiles(k):
     assert_pooled_close(g, o)
 
 
+@pytest.mark.parametrize("gh,gw", [(14, 14), (20, 20), (9, 31)])
+@pytest.mark.parametrize("k", [7, 5, 3])
+def test_van_pool_large_frames(gh, gw, k):
+    """Frames of 33 rows up to whole frames, the ones pooled on a per-warp map.
+    At 196 cells each frame goes the way that takes fewer reads (token windows
+    or separable sums); at 400 and 279 cells (more than 8 cells per lane) every
+    such frame takes the token windows. Frame sizes sweep the point where the
+    two ways cost the same for each pool size."""
+    p = gh * gw
+    H, L = 2, 1
+    rng = np.random.default_rng(7 * k + gh)
+    sizes = [33, 34, 40, 42, 43, 50, 68, 69, 100, 163, 164, p - 1, p, 37, p, 60]
+    sizes = [n for n in sizes if 33 <= n <= p]
+    pid_rows, fid_rows = [], []
+    for t, n in enumerate(sizes):
+        sel = np.sort(rng.choice(p, size=n, replace=False))
+        pid_rows.extend(sel.tolist())
+        fid_rows.extend([2 * t + 1] * n)
+    N = len(pid_rows)
+    pid = np.tile(np.array(pid_rows, np.uint16), (H, 1))
+    fid = np.tile(np.array(fid_rows, np.uint32), (H, 1))
+    van = rng.lognormal(0.0, 0.7, size=(H, N)).astype(np.float32)
+    ipv.init(device=0, dtype="bf16", max_head_dim=64, max_frame_tokens=p, max_slabs=H,
+             token_capacity=N, van_pool=True, cv_tau=(0.3, 0.9, 3.0))
+    g, ks = _run_van_pool(van, L, H, gh, gw, FORCE_POOL[k], pid, fid)
+    o, _, _ = pooled_reference(van.astype(np.float64), H, gh, gw, FORCE_POOL[k], ks, pid, fid)
+    assert list(ks) == [k]
+    assert_pooled_close(g, o)
+
+
 def test_van_pool_unaligned_layer_and_nan():
     """A layer of 45 values (the CV's scalar path) and a NaN VaN (its layer's
     CV is NaN: no pooling)."""
