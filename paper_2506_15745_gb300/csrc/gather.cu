@@ -36,7 +36,7 @@ __device__ __forceinline__ void claim_rows(const GatherArgs& a, unsigned* counte
     unsigned nxt = 0;
     if (threadIdx.x == 0) nxt = atomicAdd(counter, 1u);  // claimed ahead of need
     const int64_t b0 = static_cast<int64_t>(c) * kRowChunk;
-    dev::gather_range<CPL, kU, false, false, FIXED>(a, b0, min(total, b0 + kRowChunk), threadIdx.x >> 4,
+    dev::gather_range<CPL, kU, false, FIXED>(a, b0, min(total, b0 + kRowChunk), threadIdx.x >> 4,
                                                     blockDim.x >> 4, jn);
     __syncthreads();  // every thread has read *s_next
     if (threadIdx.x == 0) *s_next = nxt;

@@ -909,7 +909,7 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
 // slab, the kept stride staying a.budget; FIXED: the source row is
 // a.n_tokens - a.rp + j and kept is not read (the recent frames, j < rp,
 // written to rows budget - rp + j).
-template <int CPL, int kU, bool REVERSE = false, bool IDS = true, bool FIXED = false>
+template <int CPL, int kU, bool IDS = true, bool FIXED = false>
 __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begin, int64_t g_end,
                                              int64_t hw, int64_t n_hw, int64_t jn = 0) {
   const int64_t per = jn > 0 ? jn : a.budget;  // (slab, j) rows per slab in g
@@ -920,19 +920,16 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
   char* kd = static_cast<char*>(a.k_dst);
   char* vd = static_cast<char*>(a.v_dst);
 
-  // REVERSE walks the range from its end, so each slab's last rows (its
-  // recent frames, which the selection prefetches into L2) come first.
   for (int64_t g0 = g_begin + hw; g0 < g_end; g0 += n_hw * kU) {
     uint4 kr[kU][CPL], vr[kU][CPL];
     int64_t dst_off[kU];
     int src_n[kU];
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
-      const int64_t t = g0 + u * n_hw;
-      const int64_t g = REVERSE ? g_end - 1 - (t - g_begin) : t;
+      const int64_t g = g0 + u * n_hw;
       int n = -1;
       int64_t s = 0, j = 0;
-      if (t < g_end) {
+      if (g < g_end) {
         s = g / per;
         j = g - s * per;
         if (FIXED) {
