@@ -9,13 +9,14 @@
 //     value), so every block of a layer reaches the same bits and the same
 //     pool size k.
 //  2. For k > 1, each warp takes whole frames: round-robin for a cache that
-//     was never compacted, else the frames that start in its share of the
-//     rows. A frame's (VaN, 1) pairs are scattered into a dense
-//     grid_h x grid_w map in shared memory ((0, 0) where no token is cached).
-//     Window sums and counts are separable: along the grid row for every
-//     cell, then along the column; their quotient is the mean. Sums are direct (k terms each), never running sums, so a
-//     large value leaving the window cannot leave rounding behind. For k = 1
-//     the rows are copied.
+//     was never compacted, else the frames that start in the 64-row chunks
+//     it claims (pool_staged). A whole frame's (VaN, 1) pairs are scattered
+//     into a dense grid_h x grid_w map in shared memory ((0, 0) where no
+//     token is cached). Window sums and counts are separable: along the grid
+//     row for every cell, then along the column; their quotient is the mean.
+//     Sums are direct (k terms each), never running sums, so a large value
+//     leaving the window cannot leave rounding behind. For k = 1 the rows
+//     are copied.
 // Frames: rows carry (frame id, patch id) in increasing order, or derive
 // them as (n div p, n mod p) for a cache that was never compacted; a frame is
 // a maximal run of rows with one frame id.
@@ -58,13 +59,13 @@ __device__ float2 block_sum2(float2 x, float2* red) {
 }
 
 // This thread's share of sum(x - c) and sum((x - c)^2) over the layer's count
-// values (elements threadIdx.x + i * blockDim.x), eight 16-byte loads in
-// flight, fixed order. The shift c (the layer's first value) keeps the
+// values (elements threadIdx.x + i * blockDim.x), ten 16-byte loads in
+// flight (a layer of 4 x 9408 values in one round), fixed order. The shift c (the layer's first value) keeps the
 // one-sweep variance E[(x - c)^2] - E[x - c]^2 free of cancellation.
 __device__ float2 layer_sums4(const float* lv, int64_t count, float c) {
   const float4* lv4 = reinterpret_cast<const float4*>(lv);
   const int n4 = static_cast<int>(count / 4), step = blockDim.x;
-  constexpr int kU = 8;
+  constexpr int kU = 10;
   float2 a[4] = {};
   for (int i0 = threadIdx.x; i0 < n4; i0 += kU * step) {
     float4 x[kU];
@@ -301,17 +302,23 @@ __device__ void pool_tokens(const PoolArgs& pa, int p, const float* s_van, const
 
 // Phase 2 of a slab with patch and frame ids (a compacted cache): the rows
 // are staged tile by tile in shared memory; a frame (a maximal run of one
-// frame id) is pooled by the warp whose share of the tile holds its first
-// row. Frames are at most p rows long when rows are in (frame, patch) order,
-// so a tile's frames end inside its staging. Such caches hold many small
-// frames (the survivors of earlier passes): a warp takes 32 rows at a time,
-// from a frame start, and pools every frame that ends among them pairwise
-// over shuffles (same frame, within HALF rows and columns); a frame of more
-// than 32 rows goes through the map (pool_tokens).
+// frame id) is pooled by the warp that claims the chunk of kPoolChunk rows
+// holding its first row. Frames are at most p rows long when rows are in
+// (frame, patch) order, so a tile's frames end inside its staging. Such
+// caches hold many small frames (the survivors of earlier passes): a warp
+// takes 32 rows at a time, from a frame start, and pools every frame that
+// ends among them pairwise over shuffles (same frame, within HALF rows and
+// columns); a frame of more than 32 rows goes through the map (pool_tokens).
+// Chunks are claimed from a shared counter, the last rows first: the newest
+// frames, the largest and costliest, go out before the many small ones that
+// fill in behind them, so the warps finish together.
+constexpr int kPoolChunk = 64;
+
 template <int HALF>
 __device__ void pool_staged(const PoolArgs& pa, const RowIds& ids, const float* sv, float* out,
                             int n_rows, const PoolLayout& L, float* maps, const short2* ij,
                             float* s_van, uint32_t* s_fid, uint16_t* s_pid) {
+  __shared__ int s_claim;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int p = ids.p;
   float2* map = reinterpret_cast<float2*>(maps + static_cast<size_t>(warp) * L.map_floats);
@@ -319,94 +326,112 @@ __device__ void pool_staged(const PoolArgs& pa, const RowIds& ids, const float* 
     const int t1 = min(n_rows, t0 + L.tile);
     const int st0 = max(0, t0 - 1);                // one row before the tile: start detection
     const int e1 = min(n_rows, t1 + p);            // the tile's last frame ends before e1
-    __syncthreads();                               // the previous tile's staging is no longer read
-    // The first tile's ids were staged before the wait for the scores.
+    __syncthreads();                               // the previous tile's staging and claims are done
+    if (threadIdx.x == 0) s_claim = 0;
+    if (t0 == 0) {
+      // The first tile's ids were staged before the wait for the scores and
+      // its VaN while the CV was summed.
+      cp_async_wait_all();
+    } else {
 #pragma unroll 4
-    for (int m = st0 + threadIdx.x; m < e1; m += blockDim.x) {
-      s_van[m - st0] = sv[m];
-      if (t0 > 0) {
+      for (int m = st0 + threadIdx.x; m < e1; m += blockDim.x) {
+        s_van[m - st0] = sv[m];
         s_fid[m - st0] = ids.fid[m];
         s_pid[m - st0] = ids.pid[m];
       }
     }
     __syncthreads();
     if (warp >= L.nw) continue;
-    const int share = (t1 - t0 + L.nw - 1) / L.nw;
-    const int lo = t0 + warp * share;
-    const int hi = min(t1, lo + share);
-    // The first frame start at or after lo.
-    int a = hi;
-    for (int base = lo; base < hi; base += 32) {  // warp-uniform
-      const int n = base + lane;
-      const bool st = n < hi && (n == 0 || s_fid[n - st0] != s_fid[n - 1 - st0]);
-      const unsigned mask = __ballot_sync(0xffffffffu, st);
-      if (mask) {
-        a = base + __ffs(mask) - 1;
-        break;
+    const int n_chunks = (t1 - t0 + kPoolChunk - 1) / kPoolChunk;
+    for (;;) {  // warp-uniform
+      int c = 0;
+      if (lane == 0) c = atomicAdd(&s_claim, 1);
+      c = __shfl_sync(0xffffffffu, c, 0);
+      if (c >= n_chunks) break;
+      const int lo = t0 + (n_chunks - 1 - c) * kPoolChunk;
+      const int hi = min(t1, lo + kPoolChunk);
+      // The first frame start at or after lo.
+      int a = hi;
+      for (int base = lo; base < hi; base += 32) {  // warp-uniform
+        const int n = base + lane;
+        const bool st = n < hi && (n == 0 || s_fid[n - st0] != s_fid[n - 1 - st0]);
+        const unsigned mask = __ballot_sync(0xffffffffu, st);
+        if (mask) {
+          a = base + __ffs(mask) - 1;
+          break;
+        }
       }
-    }
-    while (a < hi) {  // warp-uniform; a is a frame start
-      // Rows [a, a + 32), one per lane: pool every frame that ends among them.
-      const int m = a + lane;
-      const bool valid = m < e1;
-      const uint32_t f = valid ? s_fid[m - st0] : 0u;
-      const bool st = valid && (lane == 0 || f != s_fid[m - 1 - st0]);
-      const unsigned starts = __ballot_sync(0xffffffffu, st);
-      const unsigned foreign = __ballot_sync(0xffffffffu, st && m >= hi);  // other warps' frames
-      int end;
-      if (foreign) {
-        end = __ffs(foreign) - 1;
-      } else {
-        const int nx = a + 32;
-        const bool next_starts = nx >= e1 || s_fid[nx - st0] != s_fid[nx - 1 - st0];
-        end = next_starts ? 32 : 31 - __clz(starts);  // leave a frame cut at a + 32 to the next batch
-      }
-      end = min(end, e1 - a);  // rows past the staging are not read
-      if (end == 0) {  // one frame of more than 32 rows starts at a
-        int b = e1;
-        for (int c = a + 1; c < e1; c += 32) {  // end of the run, inside the staging
-          const int mm = c + lane;
-          const unsigned other = __ballot_sync(0xffffffffu, mm < e1 && s_fid[mm - st0] != s_fid[a - st0]);
-          if (other) {
-            b = c + __ffs(other) - 1;
-            break;
+      while (a < hi) {  // warp-uniform; a is a frame start
+        // Rows [a, a + 32), one per lane: pool every frame that ends among them.
+        const int m = a + lane;
+        const bool valid = m < e1;
+        const uint32_t f = valid ? s_fid[m - st0] : 0u;
+        const bool st = valid && (lane == 0 || f != s_fid[m - 1 - st0]);
+        const unsigned starts = __ballot_sync(0xffffffffu, st);
+        const unsigned foreign = __ballot_sync(0xffffffffu, st && m >= hi);  // other warps' frames
+        int end;
+        if (foreign) {
+          end = __ffs(foreign) - 1;
+        } else {
+          const int nx = a + 32;
+          const bool next_starts = nx >= e1 || s_fid[nx - st0] != s_fid[nx - 1 - st0];
+          end = next_starts ? 32 : 31 - __clz(starts);  // leave a frame cut at a + 32 to the next batch
+        }
+        end = min(end, e1 - a);  // rows past the staging are not read
+        if (end == 0) {  // one frame of more than 32 rows starts at a
+          int b = e1;
+          for (int c = a + 1; c < e1; c += 32) {  // end of the run, inside the staging
+            const int mm = c + lane;
+            const unsigned other = __ballot_sync(0xffffffffu, mm < e1 && s_fid[mm - st0] != s_fid[a - st0]);
+            if (other) {
+              b = c + __ffs(other) - 1;
+              break;
+            }
+          }
+          pool_tokens<HALF>(pa, p, s_van, s_pid, st0, out, a, b, map, ij);
+          a = b;
+          continue;
+        }
+        // Pairwise: each lane reads the tokens of its own frame (lanes fs..fe-1
+        // of the batch) in row order; one counts when it lies within HALF grid
+        // rows and columns. The loop runs as long as the batch's longest frame.
+        // A token's grid row is offset by its frame's rank in the batch times
+        // grid_h + HALF + 1, so tokens of other frames are never within HALF
+        // rows and the loop needs no frame test; tokens without a position sit
+        // at row 0xffff, columns 8 apart. Rows stay below 2^16: grid_h <= 2005
+        // for a poolable grid, so 32 grid_h + 123 <= 64283.
+        const bool mine = lane < end;
+        const int q = mine ? s_pid[m - st0] : p;
+        const float x = mine ? s_van[m - st0] : 0.0f;
+        const bool has_pos = q < p;
+        const unsigned in_batch = starts & (end == 32 ? 0xffffffffu : ((1u << end) - 1u));
+        const unsigned upto = lane == 31 ? 0xffffffffu : ((2u << lane) - 1u);  // bits 0..lane
+        const int fs = 31 - __clz(in_batch & upto);                           // my frame's first lane
+        const unsigned after = in_batch & ~upto;
+        const int fe = after ? __ffs(after) - 1 : end;                         // one past its last lane
+        const int len = mine ? fe - fs : 0;
+        const int max_len = static_cast<int>(__reduce_max_sync(0xffffffffu, static_cast<unsigned>(len)));
+        const short2 t = has_pos ? ij[q] : make_short2(0, 0);
+        const int rank = __popc(in_batch & upto) - 1;
+        const int ti = has_pos ? t.x + rank * (pa.grid_h + HALF + 1) : 0xffff;
+        const int tj = has_pos ? t.y : lane * 8;
+        const uint32_t tij = (static_cast<uint32_t>(ti) << 16) | static_cast<uint32_t>(tj);
+        float sum = 0.0f, cnt = 0.0f;
+        for (int v = 0; v < max_len; ++v) {  // warp-uniform
+          // Lanes past fe, or wrapped below fs, hold other frames.
+          const int src = (fs + v) & 31;
+          const uint32_t tu = __shfl_sync(0xffffffffu, tij, src);
+          const float xu = __shfl_sync(0xffffffffu, x, src);
+          const unsigned du = static_cast<unsigned>(static_cast<int>(tu >> 16) - ti + HALF);
+          const unsigned dv = static_cast<unsigned>(static_cast<int>(tu & 0xffffu) - tj + HALF);
+          if (du <= 2u * HALF && dv <= 2u * HALF) {
+            sum += xu;
+            cnt += 1.0f;
           }
         }
-        pool_tokens<HALF>(pa, p, s_van, s_pid, st0, out, a, b, map, ij);
-        a = b;
-        continue;
+        if (mine) out[m] = has_pos ? __fdividef(sum, cnt) : __int_as_float(0x7fc00000);
+        a += end;
       }
-      // Pairwise: each lane reads the tokens of its own frame (lanes fs..fe-1
-      // of the batch) in row order; one counts when it lies within HALF grid
-      // rows and columns. The loop runs as long as the batch's longest frame.
-      const bool mine = lane < end;
-      const int q = mine ? s_pid[m - st0] : p;
-      const float x = mine ? s_van[m - st0] : 0.0f;
-      const bool has_pos = q < p;
-      const short2 t = has_pos ? ij[q] : make_short2(-0x4000, -0x4000);  // far from every grid cell
-      const uint32_t tij = (static_cast<uint32_t>(static_cast<uint16_t>(t.x)) << 16) |
-                           static_cast<uint16_t>(t.y);
-      const unsigned in_batch = starts & (end == 32 ? 0xffffffffu : ((1u << end) - 1u));
-      const unsigned upto = lane == 31 ? 0xffffffffu : ((2u << lane) - 1u);  // bits 0..lane
-      const int fs = 31 - __clz(in_batch & upto);                           // my frame's first lane
-      const unsigned after = in_batch & ~upto;
-      const int fe = after ? __ffs(after) - 1 : end;                         // one past its last lane
-      const int len = mine ? fe - fs : 0;
-      const int max_len = static_cast<int>(__reduce_max_sync(0xffffffffu, static_cast<unsigned>(len)));
-      float sum = 0.0f, cnt = 0.0f;
-      for (int v = 0; v < max_len; ++v) {  // warp-uniform
-        const int src = min(fs + v, 31);
-        const uint32_t tu = __shfl_sync(0xffffffffu, tij, src);
-        const float xu = __shfl_sync(0xffffffffu, x, src);
-        const int du = static_cast<int>(static_cast<int16_t>(tu >> 16)) - t.x;
-        const int dv = static_cast<int>(static_cast<int16_t>(tu & 0xffffu)) - t.y;
-        if (v < len && du >= -HALF && du <= HALF && dv >= -HALF && dv <= HALF) {
-          sum += xu;
-          cnt += 1.0f;
-        }
-      }
-      if (mine) out[m] = has_pos ? __fdividef(sum, cnt) : __int_as_float(0x7fc00000);
-      a += end;
     }
   }
 }
@@ -444,6 +469,11 @@ __global__ void __launch_bounds__(kPoolThreads, 1) pool_kernel(PoolArgs pa) {
     }
   }
   pdl_wait();  // VaN comes from the scoring kernels
+  const float* sv = pa.van + s * pa.n_tokens;
+  if (ids.fid) {  // the first tile's VaN (pool_staged) is copied while the CV is summed
+    const int e1 = min(n_rows, L.tile + p);
+    for (int m = threadIdx.x; m < e1; m += blockDim.x) cp_async4(s_van + m, sv + m);
+  }
 
   // Phase 1: CV of the layer (Algorithm 2: mu, sigma, CV = sigma / mu).
   const int64_t count = static_cast<int64_t>(pa.n_heads) * pa.n_tokens;
@@ -460,9 +490,9 @@ __global__ void __launch_bounds__(kPoolThreads, 1) pool_kernel(PoolArgs pa) {
   if (pa.pool_size && s % pa.n_heads == 0 && threadIdx.x == 0) pa.pool_size[layer] = k;
 
   // Phase 2: the pooled VaN of rows [0, n_rows) of this slab.
-  const float* sv = pa.van + s * pa.n_tokens;
   float* out = pa.pooled + s * pa.n_tokens;
   if (k == 1) {
+    cp_async_wait_all();  // no copy into shared memory outlives the block
     for (int64_t n = threadIdx.x; n < pa.n_rows; n += blockDim.x) out[n] = sv[n];
     return;
   }
