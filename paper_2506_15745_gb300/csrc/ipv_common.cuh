@@ -93,6 +93,10 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gsrc) : "memory");
 }
+// Bulk prefetch of [p, p + bytes) into L2; p 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
 // 4-byte asynchronous copy from global into shared memory (cp.async.ca);
 // both addresses 4-byte aligned.
 __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc) {

@@ -18,6 +18,7 @@ namespace ipv {
 namespace {
 
 constexpr int kScoreThreads = 768;
+constexpr int kPrefetchRows = 256;  // rows of K and of V fetched into L2 before the wait
 
 // m_q for 32/LPR patches per warp, patches flattened over (slab, q); with
 // VIRT a "slab" is a layer whose a.hs heads form one token block.
@@ -41,7 +42,6 @@ __global__ void __launch_bounds__(128) recent_mean_kernel(ScoreArgs a) {
 template <typename T, int LPR, int CPL, bool SMEM_M>
 __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(ScoreArgs a) {
   pdl_trigger();
-  pdl_wait();  // m comes from the recent-frame mean kernel
   constexpr int kU = CPL >= 4 ? 1 : 4 / CPL;
   extern __shared__ float4 sm_m4[];
   const int lane = threadIdx.x & 31;
@@ -51,6 +51,18 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(ScoreArgs a) {
   const int64_t total = a.n_slabs * n_past;
   const int64_t end = total * (blockIdx.x + 1) / gridDim.x;
   int64_t pos = total * blockIdx.x / gridDim.x;
+  if (threadIdx.x == 0 && pos < end) {
+    // K and V do not depend on the recent-frame mean: while its last blocks
+    // run, the first rows of this block's share are fetched into L2.
+    const int64_t s0 = pos / n_past;
+    const int64_t lo0 = pos - s0 * n_past;
+    const uint32_t bytes = static_cast<uint32_t>(min(min(n_past - lo0, end - pos), static_cast<int64_t>(kPrefetchRows)) *
+                                                 a.D * static_cast<int>(sizeof(T)));
+    const int64_t off = (s0 * a.cap + lo0) * a.D * static_cast<int64_t>(sizeof(T));
+    prefetch_l2(static_cast<const char*>(a.k) + off, bytes);
+    prefetch_l2(static_cast<const char*>(a.v) + off, bytes);
+  }
+  pdl_wait();  // m comes from the recent-frame mean kernel
   while (pos < end) {  // block-uniform
     const int64_t s = pos / n_past;
     const int lo = static_cast<int>(pos - s * n_past);
