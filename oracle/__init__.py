@@ -68,6 +68,8 @@ def _load():
         lib.oracle_gather_patch.restype = I32
         lib.oracle_compress.argtypes = [P, P, I32, I64, I64, I32, I64, I32, I32, I64, D,
                                         P, P, P, P, P, I32, P, I32, I32, P, P, P, I32, I32]
+        lib.oracle_uniform_select.argtypes = [I64, I64, I32, I64, P]
+        lib.oracle_uniform_select.restype = I32
         lib.oracle_frame_mean.argtypes = [P, I64, I64, I64, I32, P, I64]
         lib.oracle_frame_mean.restype = I32
         lib.oracle_scores_shared.argtypes = [P, P, I32, I64, I32, I64, I32, I64, I32, I32, P, P, P]
@@ -332,7 +334,16 @@ def compress_shared(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, gr
     return kept, kd, vd, pd, fd, ks
 
 
-ABLATIONS = {"tar_reverse": 1, "van_reverse": 2, "tar_frame": 3}
+ABLATIONS = {"tar_reverse": 1, "van_reverse": 2, "tar_frame": 3, "uniform": 4}
+
+
+def uniform_select(n_units: int, n_tokens: int, p: int, budget: int) -> np.ndarray:
+    """Uniform Select indices [n_units, budget]: the rows of budget/p whole
+    frames at regular intervals, counting back from the newest frame."""
+    kept = np.empty((n_units, budget), np.int32)
+    if _load().oracle_uniform_select(n_units, n_tokens, p, budget, _ptr(kept)) != 0:
+        raise ValueError("oracle_uniform_select rejected its arguments")
+    return kept
 
 
 def frame_mean(tar: np.ndarray, n_past: int, p: int, frame_id: np.ndarray | None = None) -> np.ndarray:
@@ -351,7 +362,7 @@ def frame_mean(tar: np.ndarray, n_past: int, p: int, frame_id: np.ndarray | None
 def compress_ablation(k: np.ndarray, v: np.ndarray, n_tokens: int, grid_h: int, grid_w: int, r: int,
                       budget: int, alpha: float, ablation: str, patch_id=None, frame_id=None):
     """Whole per-head pass with an ablation variant ("tar_reverse", "van_reverse",
-    "tar_frame"). Returns (kept, K~, V~, patch ids, frame ids)."""
+    "tar_frame", "uniform"). Returns (kept, K~, V~, patch ids, frame ids)."""
     k = np.ascontiguousarray(k)
     v = np.ascontiguousarray(v)
     S, cap, D = k.shape

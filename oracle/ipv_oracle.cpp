@@ -53,10 +53,15 @@
 // head of the layer is compacted with that layer's indices.
 //
 // Ablation variants (Sec. 4 ablation study, "TaR Reverse", "VaN Reverse",
-// "TaR Frame"), used when the pass is asked for one: a reversed stage keeps
-// the lowest scores instead of the highest (its scores negated; NaN still
-// ranks last, ties still go to the lower index); the frame-level TaR gives
-// each past token the mean TaR of the cached past tokens of its frame.
+// "TaR Frame", "Uniform Select"), used when the pass is asked for one: a
+// reversed stage keeps the lowest scores instead of the highest (its scores
+// negated; NaN still ranks last, ties still go to the lower index); the
+// frame-level TaR gives each past token the mean TaR of the cached past
+// tokens of its frame; Uniform Select (Sec. 4, KV cache compression details:
+// frames at regular intervals, all their tokens kept) ignores the scores and
+// keeps k = |C|/p whole frames of the F = |M|/p frames of the frame view,
+// every (F/k)-th frame counting back from the newest: frames
+// F - 1 - floor(i F / k), i = 0..k-1.
 //
 // Element types: bf16 (widened exactly: bits << 16) or fp32, widened to double.
 
@@ -485,6 +490,28 @@ int oracle_frame_mean(double* tar, int64_t units, int64_t n_tokens, int64_t n_pa
   return 0;
 }
 
+// Uniform Select: for each of n_units units, the rows of the k = budget / p
+// whole frames F - 1 - floor(i F / k), i = 0..k-1, of the F = n_tokens / p
+// frames (p consecutive rows each), ascending. budget must be a multiple of p
+// below n_tokens.
+int oracle_uniform_select(int64_t n_units, int64_t n_tokens, int p, int64_t budget,
+                          int32_t* kept_out) {
+  if (!kept_out || p <= 0 || n_tokens % p != 0 || budget % p != 0 || budget <= 0 ||
+      budget >= n_tokens)
+    return -1;
+  const int64_t F = n_tokens / p, k = budget / p;
+  std::vector<int64_t> frames;
+  for (int64_t i = 0; i < k; ++i) frames.push_back(F - 1 - (i * F) / k);
+  std::sort(frames.begin(), frames.end());
+  for (int64_t u = 0; u < n_units; ++u) {
+    int32_t* kept = kept_out + u * budget;
+    int64_t j = 0;
+    for (int64_t f : frames)
+      for (int q = 0; q < p; ++q) kept[j++] = static_cast<int32_t>(f * p + q);
+  }
+  return 0;
+}
+
 // One whole pass over slabs [0, n_slabs): scores, selection, compaction of K
 // and V (and of patch ids when dst_pid != NULL, of frame ids when dst_fid !=
 // NULL). With van_pool != 0 the VaN stage ranks the layer-adaptive pooled
@@ -492,7 +519,8 @@ int oracle_frame_mean(double* tar, int64_t units, int64_t n_tokens, int64_t n_pa
 // src_fid goes with src_pid). pool_size_out: [n_slabs / n_kv_heads] or NULL.
 // With shared != 0 one index set per layer is chosen (scores of the
 // concatenated head blocks) and kept_out is [n_slabs / n_kv_heads][budget].
-// ablation: 0 none, 1 TaR Reverse, 2 VaN Reverse, 3 TaR Frame.
+// ablation: 0 none, 1 TaR Reverse, 2 VaN Reverse, 3 TaR Frame, 4 Uniform
+// Select (no scores; budget a multiple of p).
 int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
                     int64_t cap, int D, int64_t n_tokens, int p, int r,
                     int64_t budget, double alpha, const uint16_t* src_pid,
@@ -507,7 +535,7 @@ int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
   const int64_t units = n_slabs / H;
   std::vector<double> tar(static_cast<size_t>(units * n_tokens));
   std::vector<double> van(tar.size());
-  if (n_tokens > budget) {
+  if (n_tokens > budget && ablation != 4) {
     const int rc = shared ? oracle_scores_shared(k, v, is_bf16, units, static_cast<int>(H), cap, D,
                                                  n_tokens, p, r, src_pid, tar.data(), van.data())
                           : oracle_scores(k, v, is_bf16, n_slabs, cap, D, n_tokens, p, r, src_pid,
@@ -539,9 +567,12 @@ int oracle_compress(const void* k, const void* v, int is_bf16, int64_t n_slabs,
     for (double& x : tar) x = -x;
   if (ablation == 2)  // VaN Reverse: the lowest VaN first
     for (double& x : van) x = -x;
-  if (oracle_select(tar.data(), van.data(), units, n_tokens, p, r, budget, alpha,
-                    kept_sel, nullptr) != 0)
+  if (ablation == 4 && n_tokens > budget) {
+    if (oracle_uniform_select(units, n_tokens, p, budget, kept_sel) != 0) return -1;
+  } else if (oracle_select(tar.data(), van.data(), units, n_tokens, p, r, budget, alpha,
+                           kept_sel, nullptr) != 0) {
     return -1;
+  }
   if (n_tokens <= budget) return 0;  // pass-through leaves the cache as it is
   // Every head of a unit is compacted with the unit's indices.
   std::vector<int32_t> kept_slab(static_cast<size_t>(n_slabs * budget));

@@ -81,6 +81,12 @@ MUTANTS = [
      "frame[n] = frame_id ? static_cast<int64_t>(frame_id[u * id_stride + n]) : 0;"),
     ("frame mean divides by the frame size p", "t[n] = a.first / static_cast<double>(a.second);",
      "t[n] = a.first / static_cast<double>(p);"),
+    ("uniform frames counted from the oldest", "frames.push_back(F - 1 - (i * F) / k);",
+     "frames.push_back((i * F) / k);"),
+    ("uniform interval rounded up", "frames.push_back(F - 1 - (i * F) / k);",
+     "frames.push_back(F - 1 - (i * F + k - 1) / k);"),
+    ("uniform keeps the first row of each frame only", "kept[j++] = static_cast<int32_t>(f * p + q);",
+     "kept[j++] = static_cast<int32_t>(f * p);"),
     ("frame ids of a fresh cache compacted as patch ids",
      "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n / p)",
      "src_fid ? src_fid[s * cap_src + n] : static_cast<uint32_t>(n % p)"),
