@@ -114,12 +114,21 @@ typedef struct {
  * still ranks last, ties still go to the lower index). TAR_FRAME: frame-level
  * redundancy, each past token's TaR replaced by the mean TaR of the cached
  * past tokens of its frame (needs frame ids once the cache holds patch ids,
- * and frame_grid_h*frame_grid_w <= IPV_MAX_POOL_FRAME_TOKENS). */
+ * and frame_grid_h*frame_grid_w <= IPV_MAX_POOL_FRAME_TOKENS). UNIFORM:
+ * "Uniform Select" (Sec. 4, KV cache compression details: frames at regular
+ * intervals, all their tokens kept), which reads no score: the n_tokens rows
+ * are F = n_tokens/p frames of p consecutive rows, and the pass keeps the
+ * k = budget/p whole frames F - 1 - floor(i F / k), i = 0..k-1 (every
+ * (F/k)-th frame counting back from the newest), in ascending row order.
+ * budget must be a multiple of p (else IPV_EINVAL); the recent-frame rule
+ * r*p < budget does not apply. Compacting whole frames keeps the cache whole
+ * frames, so a stream compressed this way stays in the frame view. */
 enum {
   IPV_ABLATION_NONE = 0,
   IPV_ABLATION_TAR_REVERSE = 1,
   IPV_ABLATION_VAN_REVERSE = 2,
-  IPV_ABLATION_TAR_FRAME = 3
+  IPV_ABLATION_TAR_FRAME = 3,
+  IPV_ABLATION_UNIFORM = 4
 };
 
 /* One tensor (K or V) of the ping-pong cache: two halves of identical

@@ -318,7 +318,7 @@ ipv_status ipv_init(const ipv_options* opt) {
   if (opt->head_shared != 0 && opt->head_shared != 1) return fail(IPV_EINVAL, "head_shared must be 0 or 1");
   if (opt->head_shared && opt->single_kernel)
     return fail(IPV_EINVAL, "head_shared runs with the step kernels only (single_kernel = 0)");
-  if (opt->ablation < IPV_ABLATION_NONE || opt->ablation > IPV_ABLATION_TAR_FRAME)
+  if (opt->ablation < IPV_ABLATION_NONE || opt->ablation > IPV_ABLATION_UNIFORM)
     return fail(IPV_EINVAL, "unknown ablation %d", opt->ablation);
   if (opt->ablation != IPV_ABLATION_NONE && opt->single_kernel)
     return fail(IPV_EINVAL, "ablation variants run with the step kernels only (single_kernel = 0)");
@@ -453,6 +453,13 @@ ipv_status ipv_select(const float* tar, const float* van, int64_t n_slabs, int64
     return after_launch(ipv::launch_passthrough(kept_idx_out, n_slabs, n_tokens, budget, st),
                         "pass-through kernel");
   if (n_tokens > IPV_MAX_TOKENS) return fail(IPV_EINVAL, "n_tokens exceeds IPV_MAX_TOKENS");
+  if (g.opt.ablation == IPV_ABLATION_UNIFORM) {  // whole frames at regular intervals; no score read
+    if (budget % p != 0) return fail(IPV_EINVAL, "Uniform Select needs a budget of whole frames");
+    prof_begin(2, st);
+    cudaError_t e = ipv::launch_uniform(kept_idx_out, n_slabs, n_tokens, static_cast<int>(p), budget, st);
+    prof_end(2, st);
+    return after_launch(e, "uniform selection kernel");
+  }
   const int64_t rp = static_cast<int64_t>(default_recent_frames(n_tokens / p)) * p;
   if (rp >= budget) return fail(IPV_EINVAL, "recent tokens r*p = %lld must be below budget", static_cast<long long>(rp));
   ipv::SelectArgs a{};
@@ -491,7 +498,11 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
                         "pass-through kernel");
   if (n_tokens > IPV_MAX_TOKENS)
     return fail(IPV_EINVAL, "n_tokens %lld exceeds IPV_MAX_TOKENS", static_cast<long long>(n_tokens));
-  if (sh.rp >= budget)
+  const bool uniform = g.opt.ablation == IPV_ABLATION_UNIFORM;
+  if (uniform && budget % sh.p != 0)
+    return fail(IPV_EINVAL, "Uniform Select needs a budget of whole frames (budget %lld, p %d)",
+                static_cast<long long>(budget), sh.p);
+  if (!uniform && sh.rp >= budget)
     return fail(IPV_EINVAL, "recent tokens r*p = %lld must be below budget %lld", static_cast<long long>(sh.rp),
                 static_cast<long long>(budget));
   if (g.opt.van_pool && k->patch_id[k->cur] && !k->frame_id[k->cur])
@@ -554,6 +565,20 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   ga.claim = g.claim;
 
   cudaError_t e;
+  if (uniform) {  // no scores: the frames' rows, then all of them through the compaction
+    prof_begin(2, st);
+    e = ipv::launch_uniform(kept_idx_out, units, sh.N, sh.p, budget, st);
+    prof_end(2, st);
+    if (e != cudaSuccess) return cuda_fail(e, "uniform selection kernel");
+    ga.rp = 0;
+    prof_begin(3, st);
+    e = ipv::launch_gather(ga, st);
+    prof_end(3, st);
+    if (e != cudaSuccess) return cuda_fail(e, "compaction kernel");
+    k->cur = 1 - k->cur;
+    v->cur = 1 - v->cur;
+    return IPV_OK;
+  }
   if (g.opt.single_kernel) {
     if (g.pipe_dirty) {
       if ((e = cudaMemsetAsync(g.pstate, 0, sizeof(ipv::PipeState), st)) != cudaSuccess ||

@@ -240,6 +240,10 @@ cudaError_t launch_passthrough(int32_t* kept, int64_t n_slabs, int64_t n_tokens,
                                cudaStream_t st);
 size_t select_smem_bytes(int64_t n_past);
 cudaError_t select_prepare(int64_t max_tokens);
+// "Uniform Select" ablation: kept [units][budget] = the rows of the budget/p
+// whole frames F - 1 - floor(i F / k) of F = n_tokens/p, ascending.
+cudaError_t launch_uniform(int32_t* kept, int64_t units, int64_t n_tokens, int p, int64_t budget,
+                           cudaStream_t st);
 
 struct GatherArgs {
   const void* k_src;

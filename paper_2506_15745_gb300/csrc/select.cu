@@ -24,7 +24,33 @@ __global__ void passthrough_kernel(int32_t* kept, int64_t n_slabs, int64_t n_tok
   }
 }
 
+// Uniform Select (Sec. 4 ablation table; frames at regular intervals, all
+// their tokens kept): element j of a unit's kept row is row q of the a-th
+// kept frame in ascending order, a = j div p, q = j mod p, whose frame is
+// F - 1 - floor((k - 1 - a) F / k). No score is read.
+__global__ void uniform_kernel(int32_t* kept, int64_t units, int64_t n_frames, int p, int64_t k) {
+  pdl_trigger();
+  const int64_t per = k * p;
+  const int64_t total = units * per;
+  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total;
+       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t j = g % per;
+    const int64_t a = j / p;
+    const int64_t f = n_frames - 1 - ((k - 1 - a) * n_frames) / k;
+    kept[g] = static_cast<int32_t>(f * p + (j - a * p));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_uniform(int32_t* kept, int64_t units, int64_t n_tokens, int p, int64_t budget,
+                           cudaStream_t st) {
+  const int64_t total = units * budget;
+  const int64_t blocks = (total + 255) / 256;
+  uniform_kernel<<<static_cast<unsigned>(blocks < 4096 ? blocks : 4096), 256, 0, st>>>(
+      kept, units, n_tokens / p, p, budget / p);
+  return cudaGetLastError();
+}
 
 size_t select_smem_bytes(int64_t n_past) {
   return dev::select_smem_words<kSelectThreads>(n_past) * sizeof(uint32_t);

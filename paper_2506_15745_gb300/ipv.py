@@ -15,7 +15,7 @@ LIB_PATH = os.path.join(_HERE, "libipv.so")
 
 IPV_OK, IPV_EINVAL, IPV_ENOINIT, IPV_ENOMEM, IPV_ECUDA, IPV_ETIMEOUT = range(6)
 IPV_BF16, IPV_F32 = 0, 1
-ABLATIONS = {"none": 0, "tar_reverse": 1, "van_reverse": 2, "tar_frame": 3}
+ABLATIONS = {"none": 0, "tar_reverse": 1, "van_reverse": 2, "tar_frame": 3, "uniform": 4}
 NUM_KERNELS = 7
 KERNEL_NAMES = ("recent_mean", "score", "select", "gather", "pipeline", "pool", "combine")
 MAX_TOKENS = 49152
@@ -130,7 +130,7 @@ def init(*, device: int = 0, dtype: str = "bf16", recent_frames: int = 0, max_he
     """ipv_init. van_pool: the VaN stage ranks layer-adaptive pooled VaN with
     pool size g(CV) from the thresholds cv_tau (Sec. 3.2, Algorithm 2).
     head_shared: one index set per layer for all its KV heads (Sec. 3.1).
-    ablation: "tar_reverse", "van_reverse" or "tar_frame" (Sec. 4 ablations)."""
+    ablation: "tar_reverse", "van_reverse", "tar_frame" or "uniform" (Sec. 4 ablations)."""
     opt = Options(device, IPV_BF16 if dtype == "bf16" else IPV_F32, recent_frames, max_head_dim,
                   max_frame_tokens, max_slabs, token_capacity, int(bool(single_kernel)),
                   int(bool(van_pool)), (ctypes.c_float * 3)(*[float(t) for t in cv_tau]),

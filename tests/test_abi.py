@@ -80,7 +80,7 @@ def test_init_option_checks(lib):
                 max_slabs=112, token_capacity=9408)
     for key, bad in [("dtype", 7), ("max_head_dim", 1024), ("max_frame_tokens", 0),
                      ("max_slabs", 0), ("token_capacity", -1), ("recent_frames", -1), ("device", -1),
-                     ("van_pool", 2), ("head_shared", 2), ("ablation", 4), ("ablation", -1)]:
+                     ("van_pool", 2), ("head_shared", 2), ("ablation", 5), ("ablation", -1)]:
         opt = ipv.Options(**dict(good, **{key: bad}))
         assert lib.ipv_init(ctypes.byref(opt)) == ipv.IPV_EINVAL, key
     tau = lambda *t: (ctypes.c_float * 3)(*t)  # noqa: E731

@@ -6,7 +6,7 @@ pass's modes: per-head index sets on the step kernels (sometimes with the
 recent-frame count overridden) or on the single persistent kernel,
 layer-adaptive pooled VaN (Sec. 3.2, Algorithm 2), one index set per layer
 (Sec. 3.1, K[:, I, :]), both of the last two, or a variant of the ablation
-table (Sec. 4). The pass runs on a fresh cache; then, twice, whole frames
+table (Sec. 4), Uniform Select included. The pass runs on a fresh cache; then, twice, whole frames
 (the AR continuation of the same streams) are appended behind the survivors,
 by torch writes or by ipv_append_frames, and it runs again on the compacted
 cache, patch and frame ids carried (Algorithm 1's loop). Every pass is
@@ -27,12 +27,13 @@ from paper_2506_15745_gb300.cache import PingPongCache  # noqa: E402
 from test_gpu_parity import check_pass, to_dev  # noqa: E402
 from test_gpu_pool import check_pooled_pass, spread_tau  # noqa: E402
 from test_gpu_ablation import _check as check_ablation_pass  # noqa: E402
+from test_gpu_ablation import check_uniform_pass  # noqa: E402
 from test_gpu_shared import check_shared_pass  # noqa: E402
 
 MODES = ("heads", "heads_single_kernel", "pooled", "shared", "shared_pooled", "tar_reverse",
-         "van_reverse", "tar_frame")
-ABLATIONS = ("tar_reverse", "van_reverse", "tar_frame")
-N_CASES = 120
+         "van_reverse", "tar_frame", "uniform")
+ABLATIONS = ("tar_reverse", "van_reverse", "tar_frame", "uniform")
+N_CASES = 135
 N_PASSES = 3
 
 
@@ -132,6 +133,8 @@ def test_random_pass_fresh_then_compacted(case):
             check_shared_pass(cache, w, N, pid_valid, tau=tau if pooled else None)
         elif pooled:
             check_pooled_pass(cache, w, N, tau, pid_valid)
+        elif ablation == "uniform":
+            check_uniform_pass(cache, w, N, pid_valid, w.n_slabs)
         elif ablation != "none":
             check_ablation_pass(cache, w, N, ablation, pid_valid)
         else:
