@@ -318,6 +318,33 @@ def test_large_config_sampled():
         torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("dtype,budget,alpha", [("bf16", 30001, 0.5), ("f32", 36864, 0.3)])
+def test_max_tokens(dtype, budget, alpha):
+    """n_tokens = IPV_MAX_TOKENS (192 frames of 16 x 16, r = 24): the largest
+    selection the library takes, with 43008 past tokens, too many for VaN to
+    sit in shared memory beside TaR, so the VaN stage reads it from L2; a
+    ragged and a whole-frame budget; then the compacted cache with 16 new
+    frames appended (patch ids carried) at the same size."""
+    S, gh, gw, D = 2, 16, 16, 128
+    p = gh * gw
+    f = ipv.MAX_TOKENS // p
+    N = f * p
+    assert N == ipv.MAX_TOKENS
+    init_for(S, N, D, p, dtype)
+    assert ipv.recent_frames(f) == 24
+    w = synth.Workload("max", 1, S, D, dtype, gh, gw, f, budget, alpha, seed=77)
+    cache = PingPongCache(S, N, D, dtype, patch_ids=True)
+    gen = synth.DeviceGenerator(w, S)  # the oracle reads the generated bytes back
+    gen.fill(cache.k[0], cache.v[0], 0, f)
+    check_pass(cache, 1, S, N, gh, gw, budget, alpha, pid_valid=False)
+    if budget % p:
+        return  # a ragged budget leaves no whole-frame cache to append to
+    n_new = (N - budget) // p
+    gen.fill(cache.k_live, cache.v_live, budget, n_new)
+    cache.pid_live[:, budget:N] = torch.arange(p, dtype=torch.int16, device="cuda").repeat(n_new)
+    check_pass(cache, 1, S, N, gh, gw, budget, alpha, pid_valid=True)
+
+
 def _run_both(w, L, make_cache, pid_valid, passes=1):
     """Run `passes` passes with the single-kernel pipeline and with the staged
     kernels on identical inputs; return both (kept, cache) results."""
