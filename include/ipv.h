@@ -51,7 +51,13 @@
  * No entry point synchronises the device or the stream, and none allocates
  * device memory except ipv_init. The library keeps one global state (device,
  * element type, scratch); calls are not thread-safe and must come from one
- * host thread at a time. Errors never trap on the device.
+ * host thread at a time. The scratch (scores, recent-frame means, the
+ * compaction's work counters) is shared by every ipv_compress and ipv_score
+ * call: two such calls whose kernels could overlap on the GPU (different
+ * streams with no event or stream order between them) race on it, so enqueue
+ * them on one stream or order them with events. ipv_select, ipv_van_pool and
+ * ipv_append_frames touch only the caller's buffers, and host-device copies
+ * on other streams may overlap any call. Errors never trap on the device.
  */
 #ifndef IPV_H_
 #define IPV_H_

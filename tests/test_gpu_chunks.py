@@ -47,3 +47,31 @@ def test_layer_chunks_equal_the_whole_pass(shared):
     for a, b in zip(*outs):
         assert torch.equal(a, b)
     assert (outs[0][0] >= 0).all()
+
+
+def test_pass_on_a_side_stream():
+    """The pass enqueued on a non-default stream (inputs written on that
+    stream, the result read after synchronising it) equals the pass on the
+    default stream bit for bit: every kernel of the call follows the given
+    stream."""
+    w = synth.CONFIGS["llava"].scaled(n_layers=3, n_kv_heads=4, head_dim=128, grid_h=7, grid_w=7,
+                                      n_frames=16, budget=10 * 49, seed=9)
+    S, N, C, D = w.n_slabs, w.n_tokens, w.budget, w.head_dim
+    ipv.init(device=0, dtype=w.dtype, max_head_dim=D, max_frame_tokens=w.p, max_slabs=S,
+             token_capacity=N)
+    outs = []
+    for use_side in (False, True):
+        st = torch.cuda.Stream() if use_side else torch.cuda.current_stream()
+        with torch.cuda.stream(st):
+            cache = PingPongCache(S, N, D, w.dtype, patch_ids=True)
+            synth.device_generate(w, cache.k[0], cache.v[0])
+            cache.n_tokens = N
+            kept = torch.full((S, C), -1, dtype=torch.int32, device="cuda")
+            cache.compress(w.n_layers, w.n_kv_heads, w.grid_h, w.grid_w, C, w.tar_ratio, kept,
+                           pid_valid=False, stream=st)
+        st.synchronize()
+        outs.append((kept.clone(), cache.k_live[:, :C].clone(), cache.v_live[:, :C].clone(),
+                     cache.pid_live[:, :C].clone()))
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+    assert (outs[0][0] >= 0).all()

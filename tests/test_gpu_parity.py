@@ -141,6 +141,8 @@ EDGE_CASES = [
     (1, 9, 1, 1, 64, "bf16", lambda N, p, rp: 4, 0.5),                    # p = 1
     (2, 8, 4, 4, 64, "f32", lambda N, p, rp: N, 0.5),                     # pass-through N == C
     (2, 8, 4, 4, 64, "f32", lambda N, p, rp: N + 9, 0.5),                 # pass-through N < C
+    (2, 9, 20, 20, 128, "bf16", lambda N, p, rp: 5 * p + 17, 0.5),        # m table > 200 KB: read via L2
+    (1, 8, 9, 12, 512, "f32", lambda N, p, rp: 3 * p, 0.7),              # the same at 2 KB rows
 ]
 
 
