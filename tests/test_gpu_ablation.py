@@ -40,7 +40,9 @@ def _shutdown_after():
     ipv.shutdown()
 
 
-def _check(cache, w, N, variant, pid_valid):
+def check_ablation_pass(cache, w, N, variant, pid_valid):
+    """One pass of a score-ranking variant on live rows 0..N-1, checked against
+    the oracle on the scores that variant ranks."""
     L, H, D, gh, gw, B, p = w.n_layers, w.n_kv_heads, w.head_dim, w.grid_h, w.grid_w, w.budget, w.p
     r = ipv.recent_frames(N // p)
     n_past = N - r * p
@@ -91,12 +93,12 @@ def test_ablation_fresh_then_compacted(variant, dtype):
     cache.v.zero_()
     cache.k[0] = to_dev(K[:, :N], dtype)
     cache.v[0] = to_dev(V[:, :N], dtype)
-    _check(cache, w, N, variant, pid_valid=False)
+    check_ablation_pass(cache, w, N, variant, pid_valid=False)
     c = cache.cur
     k, v = cache.structs(pid_valid=True)
     ipv.append_frames(k, v, to_dev(K[:, N:N + 6 * p], dtype), to_dev(V[:, N:N + 6 * p], dtype),
                       w.n_layers, w.n_kv_heads, w.head_dim, B, 6, w.grid_h, w.grid_w)
-    _check(cache, w, N, variant, pid_valid=True)
+    check_ablation_pass(cache, w, N, variant, pid_valid=True)
 
 
 def test_tar_frame_needs_frame_ids_with_patch_ids():

@@ -6,10 +6,11 @@ pass's modes: per-head index sets on the step kernels (sometimes with the
 recent-frame count overridden) or on the single persistent kernel,
 layer-adaptive pooled VaN (Sec. 3.2, Algorithm 2), one index set per layer
 (Sec. 3.1, K[:, I, :]), both of the last two, or a variant of the ablation
-table (Sec. 4), Uniform Select included. The pass runs on a fresh cache; then, twice, whole frames
-(the AR continuation of the same streams) are appended behind the survivors,
-by torch writes or by ipv_append_frames, and it runs again on the compacted
-cache, patch and frame ids carried (Algorithm 1's loop). Every pass is
+table (Sec. 4), Uniform Select included. The pass runs on a fresh cache;
+then, twice, whole frames (the AR continuation of the same streams) are
+appended behind the survivors, by torch writes or by ipv_append_frames, and
+it runs again on the compacted cache, patch and frame ids carried
+(Algorithm 1's loop). Every pass is
 checked against the oracle with the rules of parity.py: scores, pooled
 scores and pool sizes, indices, compacted bytes and ids.
 """
@@ -26,7 +27,7 @@ from paper_2506_15745_gb300 import ipv  # noqa: E402
 from paper_2506_15745_gb300.cache import PingPongCache  # noqa: E402
 from test_gpu_parity import check_pass, to_dev  # noqa: E402
 from test_gpu_pool import check_pooled_pass, spread_tau  # noqa: E402
-from test_gpu_ablation import _check as check_ablation_pass  # noqa: E402
+from test_gpu_ablation import check_ablation_pass  # noqa: E402
 from test_gpu_ablation import check_uniform_pass  # noqa: E402
 from test_gpu_shared import check_shared_pass  # noqa: E402
 
