@@ -39,6 +39,8 @@ def workload_desc(w: synth.Workload) -> str:
         d += f", layer-adaptive pooled VaN (CV thresholds {tuple(w.cv_tau)})"
     if w.head_shared:
         d += ", one index set per layer shared by its KV heads"
+    if w.ablation != "none":
+        d += f", ablation variant {w.ablation}"
     return d
 
 
@@ -83,6 +85,10 @@ def bytes_model(w: synth.Workload, S: int, r: int):
         per_kernel["gather"] = S * 4 * C * row + L * 4 * C
         if w.van_pool:
             per_kernel["pool"] = L * (4 * N + 4 * n_past)
+    if w.ablation == "uniform":
+        # Uniform Select reads no score: kept indices out, the kept rows copied
+        pass_bytes = tight = S * row * 4 * C + S * C * 4
+        per_kernel.update(recent_mean=0, score=0, select=S * 4 * C, pool=0, combine=0)
     return pass_bytes, tight, per_kernel
 
 
@@ -90,6 +96,9 @@ def oracle_pass(w: synth.Workload, k_np, v_np, r: int):
     """One oracle pass over the given slabs (pooled VaN if the workload asks
     for it; then the slabs are whole layers)."""
     import oracle
+    if w.ablation != "none":
+        return oracle.compress_ablation(k_np, v_np, w.n_tokens, w.grid_h, w.grid_w, r, w.budget,
+                                        w.tar_ratio, w.ablation)
     if w.head_shared:
         return oracle.compress_shared(k_np, v_np, w.n_tokens, w.grid_h, w.grid_w, r, w.budget,
                                       w.tar_ratio, w.n_kv_heads,
@@ -434,14 +443,15 @@ def run_stream(args, w: synth.Workload):
     S, N, C, D, p = w.slabs_per_stream, w.n_tokens, w.budget, w.head_dim, w.p
     ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
              token_capacity=N, single_kernel=args.single_kernel, van_pool=w.van_pool,
-             cv_tau=w.cv_tau, head_shared=w.head_shared)
+             cv_tau=w.cv_tau, head_shared=w.head_shared, ablation=w.ablation)
     r = ipv.recent_frames(w.n_frames)
     kept = torch.empty((S // w.n_kv_heads if w.head_shared else S, C), dtype=torch.int32,
                        device="cuda")
     pid_block = torch.arange(w.append_frames * p, device="cuda").remainder(p).to(torch.int16)
 
     def stream(timed: bool, profile_passes: int = 0):
-        cache = PingPongCache(S, N, D, w.dtype, patch_ids=True, frame_ids=w.van_pool)
+        cache = PingPongCache(S, N, D, w.dtype, patch_ids=True,
+                              frame_ids=w.van_pool or w.ablation == "tar_frame")
         gen = synth.DeviceGenerator(w, S, stream=rank)
         evs, frames, n_pass = [], 0, 0
         t0 = torch.cuda.Event(enable_timing=True)
@@ -579,7 +589,7 @@ def run_gpu(args, w: synth.Workload):
 
     ipv.init(device=local, dtype=w.dtype, max_head_dim=D, max_frame_tokens=p, max_slabs=S,
              token_capacity=N, single_kernel=args.single_kernel, van_pool=w.van_pool,
-             cv_tau=w.cv_tau, head_shared=w.head_shared)
+             cv_tau=w.cv_tau, head_shared=w.head_shared, ablation=w.ablation)
     r = ipv.recent_frames(w.n_frames)
     cache = PingPongCache(S, N, D, w.dtype, patch_ids=False)
     for i, st in enumerate(streams):
@@ -725,6 +735,9 @@ def main(argv=None):
     ap.add_argument("--graph-steps", type=int, default=100,
                     help="streaming configs: steady-state steps timed eager and as CUDA-graph replays")
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    ap.add_argument("--ablation", default="none",
+                    choices=["none", "tar_reverse", "van_reverse", "tar_frame", "uniform"],
+                    help="run a variant of the ablation table (Sec. 4) on the chosen workload")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--e2e-max-gb", type=float, default=8.0)
     ap.add_argument("--prof-steps", type=int, default=200)
@@ -735,6 +748,10 @@ def main(argv=None):
                     help="run the pass as one persistent kernel instead of the step kernels")
     args = ap.parse_args(argv)
     w = synth.CONFIGS[args.config]
+    if args.ablation != "none":  # a variant of the ablation table on the same workload
+        if w.van_pool or w.head_shared:
+            ap.error("--ablation runs on the per-head, raw-VaN workloads")
+        w = w.scaled(name=f"{w.name}+{args.ablation}", ablation=args.ablation)
     if args.impl == "reference":
         run_reference(args, w)
     elif w.stream_frames:

@@ -64,6 +64,7 @@ class Workload:
     van_pool: bool = False                 # layer-adaptive VaN pooling in the pass
     cv_tau: tuple = (0.0, 0.0, 0.0)        # CV thresholds of the pool-size map
     head_shared: bool = False              # one index set per layer for all its KV heads
+    ablation: str = "none"                 # a variant of the ablation table for the pass
 
     @property
     def p(self) -> int:
