@@ -238,6 +238,25 @@ def test_invalid_arguments_are_rejected():
         assert k.cur == 0 and v.cur == 0
 
 
+def test_scratch_allocation_failure_is_reported_and_recovered():
+    """ipv_init asking for more scratch than the GPU holds fails with
+    IPV_ENOMEM (no kernel runs, nothing stays allocated), leaves the library
+    uninitialised, and the next ipv_init and pass work as before."""
+    slabs, cap = 2_000_000, 49152  # 393 GB per score array
+    free, total = torch.cuda.mem_get_info()
+    assert slabs * cap * 4 > total
+    with pytest.raises(ipv.IpvError) as ei:
+        ipv.init(device=0, dtype="bf16", max_head_dim=128, max_frame_tokens=256, max_slabs=slabs,
+                 token_capacity=cap)
+    assert ei.value.status == ipv.IPV_ENOMEM
+    assert ipv.recent_frames(48) == -1  # not initialised
+    assert torch.cuda.mem_get_info()[0] >= free - (64 << 20)  # the partial allocations were freed
+    S, f, gh, gw, D = 2, 10, 4, 5, 64
+    init_for(S, f * gh * gw, D, gh * gw, "bf16")
+    cache = host_case(S, f, gh, gw, D, "bf16", seed=12)
+    check_pass(cache, 1, S, f * gh * gw, gh, gw, 90, 0.5, pid_valid=False)
+
+
 def _device_config(name, patch_ids=False):
     w = synth.CONFIGS[name]
     init_for(w.slabs_per_stream, w.n_tokens, w.head_dim, w.p, w.dtype)
