@@ -735,6 +735,8 @@ def main(argv=None):
     ap.add_argument("--graph-steps", type=int, default=100,
                     help="streaming configs: steady-state steps timed eager and as CUDA-graph replays")
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    ap.add_argument("--seed", type=int, default=None,
+                    help="seed of the synthetic inputs (default: the workload's own)")
     ap.add_argument("--ablation", default="none",
                     choices=["none", "tar_reverse", "van_reverse", "tar_frame", "uniform"],
                     help="run a variant of the ablation table (Sec. 4) on the chosen workload")
@@ -748,6 +750,8 @@ def main(argv=None):
                     help="run the pass as one persistent kernel instead of the step kernels")
     args = ap.parse_args(argv)
     w = synth.CONFIGS[args.config]
+    if args.seed is not None:
+        w = w.scaled(seed=args.seed)
     if args.ablation != "none":  # a variant of the ablation table on the same workload
         if w.van_pool or w.head_shared:
             ap.error("--ablation runs on the per-head, raw-VaN workloads")
