@@ -27,21 +27,35 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "compress-pass latency (ms) and HBM GB/s vs GB300 peak, 7B shape 6K budget"
-KERNELS = ("recent_mean", "score", "select", "gather", "pipeline", "pool", "combine")
+KERNELS = ("recent_mean", "score", "select", "gather", "fused", "pool", "combine")
 FALLBACK_HBM_GBS = 6800.0
 
 
 def workload_desc(w: synth.Workload) -> str:
-    d = (f"{w.name}: {w.n_streams}x{w.n_layers} layers x {w.n_kv_heads} KV heads x "
-         f"head_dim {w.head_dim} {w.dtype}, {w.grid_h}x{w.grid_w} tokens/frame, "
-         f"{w.n_frames} frames ({w.n_tokens} tokens) -> budget {w.budget}, alpha {w.tar_ratio}")
+    """The workload in under 120 characters (the options go in config keys)."""
+    return (f"{w.name}: {w.n_streams}x{w.n_layers}L x {w.n_kv_heads} KV heads x {w.head_dim} {w.dtype}, "
+            f"{w.grid_h}x{w.grid_w}/frame, {w.n_frames} frames ({w.n_tokens} tok) -> {w.budget}, "
+            f"alpha {w.tar_ratio}")
+
+
+def workload_options(w: synth.Workload) -> dict:
+    opts = {}
     if w.van_pool:
-        d += f", layer-adaptive pooled VaN (CV thresholds {tuple(w.cv_tau)})"
+        opts["van"] = f"layer-adaptive pooled, CV thresholds {tuple(w.cv_tau)}"
     if w.head_shared:
-        d += ", one index set per layer shared by its KV heads"
+        opts["index_set"] = "one per layer, shared by its KV heads"
     if w.ablation != "none":
-        d += f", ablation variant {w.ablation}"
-    return d
+        opts["ablation"] = w.ablation
+    return opts
+
+
+def run_config(w: synth.Workload, S: int, r: int, world: int, n_streams: int) -> dict:
+    """The config object of a bench line; both arms print the same one."""
+    return {"workload": workload_desc(w), **workload_options(w), "storage_dtype": w.dtype,
+            "streams_per_gpu": n_streams, "slabs_per_gpu": S, "recent_frames": r,
+            "l2": "flushed (256 MiB write) before every timed pass; inputs "
+                  f"{2 * S * w.n_tokens * w.head_dim * w.elem_bytes / 1e6:.0f} MB > L2",
+            "parallelism": f"independent streams, {world} GPU(s), no collective"}
 
 
 def peaks():
@@ -66,7 +80,7 @@ def bytes_model(w: synth.Workload, S: int, r: int):
         "score": S * (2 * n_past * row + 8 * n_past),
         "select": S * (8 * n_past + 4 * C),
         "gather": S * (4 * C * row + 4 * C),
-        "pipeline": pass_bytes,  # the single-kernel pass does all four steps
+        "fused": pass_bytes,  # the fused pass does all four steps
         "pool": 0,
         "combine": 0,
     }
@@ -212,39 +226,70 @@ def time_oracle(w: synth.Workload, k_np, v_np, r: int, budget_s: float = 12.0):
     return ms_pass, n, dt
 
 
+def _host_part(args):
+    w, s0, s1 = args
+    return synth.host_generate(w, slabs=s1 - s0, slab0=s0)
+
+
+def host_inputs(w: synth.Workload, S: int):
+    """K, V of the first S slabs of stream 0, generated on the host by a pool
+    of processes (spawned: no forked copy of an initialised runtime)."""
+    import concurrent.futures as cf
+    import multiprocessing as mp
+    n_proc = max(1, min(len(os.sched_getaffinity(0)), 16, S))
+    bounds = [(S * i // n_proc, S * (i + 1) // n_proc) for i in range(n_proc)]
+    if n_proc == 1:
+        return synth.host_generate(w, slabs=S)
+    with cf.ProcessPoolExecutor(n_proc, mp_context=mp.get_context("spawn")) as ex:
+        parts = list(ex.map(_host_part, [(w, a, b) for a, b in bounds]))
+    return np.concatenate([k for k, _ in parts]), np.concatenate([v for _, v in parts])
+
+
 def run_reference(args, w: synth.Workload):
-    """The reference arm: the CPU oracle as it stands, on host cores, rank 0 only."""
+    """The reference arm: the CPU oracle as it stands, on host cores, rank 0
+    only. A step is one whole pass over every slab of one stream, as the GPU
+    arm's; only if K + W such passes would not end within --ref-seconds does a
+    step take the first slabs only, and the line says so."""
     world, rank, _ = dist_setup()
     if rank != 0:
         return
     import oracle
     oracle.build()
+    from paper_2506_15745_gb300.shard import shard_range
     r = oracle.recent_frames(w.n_frames)
     unit = w.n_kv_heads if (w.van_pool or w.head_shared) else 1  # whole layers
+    # The slabs one GPU's pass covers, as in the GPU arm: rank 0's share of
+    # the streams of a multi-stream workload, else one stream.
+    n_str = 1
+    if w.n_streams > 1:
+        s0, s1 = shard_range(w.n_streams, 0, world)
+        n_str = s1 - s0
+    S = w.slabs_per_stream * n_str
     K1, V1 = synth.host_generate(w.scaled(n_streams=1), slabs=unit)
     t0 = time.perf_counter()
     oracle_pass(w, K1, V1, r)
     t_slab = (time.perf_counter() - t0) / unit
-    # Slabs per step: at most --ref-slabs, fewer if the run would exceed ~2 min.
-    fit = int(120.0 / max(1e-6, (args.steps + args.warmup) * t_slab))
-    per_step_slabs = max(1, min(w.slabs_per_stream, args.ref_slabs, fit))
-    per_step_slabs = max(unit, per_step_slabs // unit * unit)
-    K, V = synth.host_generate(w.scaled(n_streams=1), slabs=per_step_slabs)
+    fit = int(args.ref_seconds / max(1e-6, (args.steps + args.warmup) * t_slab))
+    per_step_slabs = max(unit, min(S, w.slabs_per_stream, fit) // unit * unit)
+    K, V = host_inputs(w.scaled(n_streams=1), per_step_slabs)
     for _ in range(args.warmup):
-        oracle_pass(w, K[:unit], V[:unit], r)
+        oracle_pass(w, K, V, r)
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
         oracle_pass(w, K, V, r)
         times.append(time.perf_counter() - t0)
-    ms = float(np.mean(times)) * 1e3 * w.n_slabs / per_step_slabs
-    sample = (f"{per_step_slabs} of {w.n_slabs} slabs per step (host-generated, same recipe), "
-              f"extrapolated x{w.n_slabs / per_step_slabs:.1f} to a full pass")
+    ms = float(np.mean(times)) * 1e3 * S / per_step_slabs
+    if per_step_slabs == S:
+        sample = f"every one of the {S} slabs of the pass in every step (host-generated, same recipe)"
+    else:
+        sample = (f"{per_step_slabs} of {S} slabs per step (host-generated, same recipe), "
+                  f"extrapolated x{S / per_step_slabs:.1f} to a full pass")
     line = {
         "impl": "reference", "metric": METRIC, "value": ms, "unit": "ms", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": workload_desc(w)},
+        "data": "synthetic", "config": run_config(w, S, r, world, n_str),
         "cpu_baseline": {"value": ms, "unit": "ms", "cores": 1, "kind": "oracle", "sample": sample},
         "e2e": {"value": ms, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -528,13 +573,13 @@ def run_stream(args, w: synth.Workload):
             "steps": len(evs), "warmup": max(1, args.warmup // 10), "ms_per_step": float(per_pass.mean()),
             "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
-            "config": {"workload": workload_desc(w) + f", streamed: {w.stream_frames} frames, "
-                                                       f"{w.append_frames} appended per step",
+            "config": {"workload": workload_desc(w), **workload_options(w),
+                       "stream": f"{w.stream_frames} frames, {w.append_frames} appended per step",
                        "storage_dtype": w.dtype, "streams_per_gpu": 1, "slabs_per_gpu": S,
                        "recent_frames": r,
                        "l2": "not flushed: each pass follows the appends, as in deployment",
                        "parallelism": f"independent streams, {world} GPU(s), no collective"},
-            "path": "single-kernel pipeline" if args.single_kernel else "step kernels",
+            "path": "fused single kernel" if args.single_kernel else "step kernels",
             "passes": len(evs),
             "per_pass_ms_p50": p50, "per_pass_ms_p99": p99,
             "per_pass_ms_mean": float(per_pass.mean()), "per_pass_ms_max": float(per_pass.max()),
@@ -688,12 +733,7 @@ def run_gpu(args, w: synth.Workload):
             "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_pass_max,
             "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
-            "config": {"workload": workload_desc(w), "storage_dtype": w.dtype,
-                       "streams_per_gpu": len(streams), "slabs_per_gpu": S,
-                       "recent_frames": r,
-                       "l2": "flushed (256 MiB write) before every timed pass; inputs "
-                             f"{2 * S * N * D * w.elem_bytes / 1e6:.0f} MB > L2",
-                       "parallelism": f"independent streams, {world} GPU(s), no collective"},
+            "config": run_config(w, S, r, world, len(streams)),
             "pass_bytes": pass_bytes,
             "pass_gbs": pass_bytes / (ms_pass_max * 1e-3) / 1e9,
             "pass_roofline_frac": pass_bytes / (ms_pass_max * 1e-3) / 1e9 / peak,
@@ -703,7 +743,7 @@ def run_gpu(args, w: synth.Workload):
             "per_pass_ms_p99": float(np.percentile(per_pass, 99)),
             "kernel_ms": {k: round(kern_ms[k], 5) for k in KERNELS},
             "kernel_ms_source": f"CUDA events around each kernel over {prof_steps} further passes",
-            "path": "single-kernel pipeline" if args.single_kernel else "step kernels",
+            "path": "fused single kernel" if args.single_kernel else "step kernels",
             "dram_min_bytes": dram_min_bytes(w, S, r),
             "dram_min_frac": dram_min_bytes(w, S, r) / (ms_pass_max * 1e-3) / 1e9 / peak,
             "roofline": {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": peak,
@@ -745,9 +785,10 @@ def main(argv=None):
     ap.add_argument("--prof-steps", type=int, default=200)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--ref-slabs", type=int, default=4)
+    ap.add_argument("--ref-seconds", type=float, default=150.0,
+                    help="reference arm: time budget of its K + W oracle passes")
     ap.add_argument("--single-kernel", action="store_true",
-                    help="run the pass as one persistent kernel instead of the step kernels")
+                    help="run the pass as the fused persistent kernel instead of the step kernels")
     args = ap.parse_args(argv)
     w = synth.CONFIGS[args.config]
     if args.seed is not None:

@@ -90,8 +90,15 @@ typedef struct {
   int64_t token_capacity; /* rows per slab in each cache half (the slab stride) */
   int single_kernel;      /* 0: ipv_compress runs the pass as its four step kernels
                              (recent-frame mean, scoring, selection, compaction),
-                             one after the other; 1: as one persistent kernel whose
-                             blocks overlap the steps of different slabs. Both give
+                             one after the other; 1: as one fused persistent kernel
+                             (cooperative launch, two blocks per SM) that works
+                             through the slabs in order and compacts each slab a few
+                             slabs after scoring it, so that its kept rows are read
+                             from L2 instead of HBM. The fused kernel takes caches
+                             that have never been compacted (the live half has no
+                             patch ids) and whose selection keys fit the registers
+                             of one block (n_tokens - r*p <= 9216 past tokens);
+                             other calls run the step kernels. Both give
                              bit-identical results. */
   int van_pool;           /* 0: the VaN stage ranks raw VaN (Sec. 3.2 s_VaN);
                              1: it ranks layer-adaptive pooled VaN (Sec. 3.2,
@@ -274,7 +281,7 @@ const char* ipv_status_string(ipv_status s);
 /* Kernel timing for benchmarks: while enabled, ipv_compress and ipv_score
  * record CUDA events around each kernel on the call's stream. Kernel ids:
  * 0 recent-frame mean, 1 scoring, 2 selection, 3 compaction, 4 the
- * single-kernel pass, 5 VaN pooling, 6 the per-layer combination of head
+ * fused pass (single_kernel = 1), 5 VaN pooling, 6 the per-layer combination of head
  * sums (head_shared). The frame-level TaR kernel of the TAR_FRAME ablation
  * is not timed. */
 #define IPV_NUM_KERNELS 7
@@ -303,7 +310,9 @@ ipv_status ipv_profile_collect(double ms_out[IPV_NUM_KERNELS],
  * A pass that needs more is rejected with IPV_EINVAL before anything is
  * enqueued (the LLaVA-OV-7B and Qwen2-VL-7B shapes fit).
  * The first call on a device sets that device up once (kernel limits and
- * cudaGetSymbolAddress of the array): make it before any stream capture. All
+ * cudaGetSymbolAddress of the array): make it before any stream capture. That
+ * set-up is kept until the process exits, so resetting the device
+ * (cudaDeviceReset) after the first call is not supported. All
  * calls on a device share the array, so calls that may overlap on the GPU
  * race and must be ordered by the caller. Errors: as ipv_compress, plus
  * IPV_EINVAL for a pass too large for the array. */
@@ -313,18 +322,19 @@ ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype, int64_t to
                                int64_t n_tokens, int frame_grid_h, int frame_grid_w, int64_t budget,
                                float tar_ratio, int32_t* kept_idx_out, void* stream);
 
-/* Diagnostic: the single-kernel pass bounds every wait and, when one runs
- * out, sets bits in a device error word (1: a score chunk gave up waiting for
- * its slab's recent-frame mean; 2: a block gave up waiting for work). This
- * waits for the whole device, copies the word to *err_out (0 = no timeout
- * since the last read) and clears it. Errors: IPV_ENOINIT, IPV_EINVAL, IPV_ECUDA. */
+/* Diagnostic: the fused pass (single_kernel = 1) bounds every wait and, when
+ * one runs out, sets bits in a device error word (1: a block gave up waiting
+ * for its slab's scores before the selection; 2: a block gave up waiting for
+ * a slab's selection before compacting it). This waits for the whole device,
+ * copies the word to *err_out (0 = no timeout since the last read) and clears
+ * it. Errors: IPV_ENOINIT, IPV_EINVAL, IPV_ECUDA. */
 ipv_status ipv_device_error(uint32_t* err_out);
 
-/* Diagnostic: the number of polls after which each wait of the single-kernel
+/* Diagnostic: the number of polls after which each wait of the fused
  * pass gives up (0 restores the default, 2^20 polls of about 0.1-0.3 us). A
  * wait that gives up sets its bit in the device error word and the pass goes
  * on without the awaited data: its results are then invalid, the device
- * stays usable, and the next pass starts from a clean queue state. A short
+ * stays usable, and the next pass starts from clean counters. A short
  * limit makes a pass fail fast instead of waiting; tests use it to exercise
  * the error path. Takes effect at the next ipv_compress. Errors:
  * IPV_EINVAL (negative), IPV_ENOINIT. */

@@ -15,7 +15,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJ = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libipv.so")
-SOURCES = ["api.cu", "score.cu", "select.cu", "gather.cu", "pool.cu", "combine.cu", "append.cu", "pipeline.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "score.cu", "select.cu", "gather.cu", "pool.cu", "combine.cu", "append.cu", "window.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

@@ -1,6 +1,7 @@
 // C ABI of libipv.so (declared in include/ipv.h): state, argument checks,
 // kernel sequencing and optional per-kernel event timing.
 #include <cmath>
+#include <cstddef>
 #include <cstdarg>
 #include <cstdio>
 #include <ctime>
@@ -30,11 +31,11 @@ struct State {
   float* kk = nullptr;      // [max_slabs][token_capacity], head_shared only: per-head |k|^2
   float* tar_l = nullptr;   // [max_slabs][token_capacity], head_shared only: per-layer scores
   float* van_l = nullptr;
-  ipv::PipeState* pstate = nullptr;
-  unsigned* pflags = nullptr;  // [kPipeFlags][max_slabs]
+  ipv::WinState* wstate = nullptr;
+  unsigned* wflags = nullptr;  // [kWinFlags][max_slabs]
   unsigned* claim = nullptr;   // [3] compaction work counters, zero between passes
-  bool pipe_dirty = false;     // a failed launch may have left queue state behind
-  int64_t wait_limit = int64_t{1} << 20;  // polls before a wait of the single-kernel pass gives up
+  bool win_dirty = false;      // a failed launch may have left counters behind
+  int64_t wait_limit = int64_t{1} << 20;  // polls before a wait of the fused pass gives up
   bool profiling = false;
   std::vector<EventPair> pool;                      // idle event pairs
   std::vector<EventPair> pending[IPV_NUM_KERNELS];  // recorded, not yet read
@@ -46,7 +47,7 @@ thread_local std::string g_err;
 void free_scratch(State& s) {
   for (void* p : {static_cast<void*>(s.tar), static_cast<void*>(s.van), static_cast<void*>(s.m),
                   static_cast<void*>(s.pooled), static_cast<void*>(s.kk), static_cast<void*>(s.tar_l),
-                  static_cast<void*>(s.van_l), static_cast<void*>(s.pstate), static_cast<void*>(s.pflags),
+                  static_cast<void*>(s.van_l), static_cast<void*>(s.wstate), static_cast<void*>(s.wflags),
                   static_cast<void*>(s.claim)})
     cudaFree(p);
 }
@@ -269,6 +270,57 @@ cudaError_t launch_shared_scores(const ipv::ScoreArgs& phys, int n_kv_heads, flo
   return e;
 }
 
+// Work decomposition of the fused pass (window.cu). Tuning constants: score
+// items of at most kWinPatches patches, gather items of kWinRows selected
+// rows, and a lag of kWinLag slabs between a slab's score and gather items.
+#ifndef IPV_WIN_PATCHES
+#define IPV_WIN_PATCHES 16
+#endif
+#ifndef IPV_WIN_ROWS
+#define IPV_WIN_ROWS 512
+#endif
+#ifndef IPV_WIN_LAG
+#define IPV_WIN_LAG 4
+#endif
+
+size_t fused_smem(const ipv::WinArgs& w) {
+  return ipv::window_smem_bytes(w.qmax, w.sc.D, w.sc.is_bf16 ? 2 : 4, w.sc.r,
+                                w.sc.n_tokens - static_cast<int64_t>(w.sc.r) * w.sc.p);
+}
+
+// Fills the fused pass's arguments; false if the pass does not fit it (the
+// selection's keys in the registers of one block, a score item's recent rows
+// in shared memory that leaves room for a second block on the SM).
+bool fused_args(const ipv::ScoreArgs& a, const ipv::SelectArgs& sa, const ipv::GatherArgs& ga,
+                const Shape& sh, int64_t budget, ipv::WinArgs* w) {
+  const int64_t n_past = sh.N - sh.rp;
+  if (n_past > static_cast<int64_t>(ipv::kWinBlock) * ipv::kWinRegE) return false;
+  w->sc = a;
+  w->se = sa;
+  w->ga = ga;
+  w->state = g.wstate;
+  w->flags = g.wflags;
+  w->n_si = (sh.p + IPV_WIN_PATCHES - 1) / IPV_WIN_PATCHES;
+  w->qmax = (sh.p + w->n_si - 1) / w->n_si;
+  while (w->qmax > 1 && fused_smem(*w) > ipv::kWinSmemMax) {  // fewer patches per item for wide rows
+    w->n_si = (sh.p + w->qmax - 2) / (w->qmax - 1);
+    w->qmax = (sh.p + w->n_si - 1) / w->n_si;
+  }
+  w->rows_gi = IPV_WIN_ROWS;
+  w->n_gi = static_cast<int>((budget - sh.rp + IPV_WIN_ROWS - 1) / IPV_WIN_ROWS);
+  w->lag = IPV_WIN_LAG;
+  w->n_stream = g.num_sms;
+  w->n_owner = static_cast<int>(sh.S < g.num_sms ? sh.S : g.num_sms);
+  w->spin_limit = g.wait_limit;
+  if (fused_smem(*w) > ipv::kWinSmemMax) return false;
+  int per_sm = 0;
+  if (ipv::window_blocks_per_sm(*w, fused_smem(*w), &per_sm) != cudaSuccess || per_sm < 2) {
+    cudaGetLastError();
+    return false;
+  }
+  return true;
+}
+
 }  // namespace
 
 namespace ipv {
@@ -344,7 +396,7 @@ ipv_status ipv_init(const ipv_options* opt) {
   if ((e = ipv::score_prepare(opt->max_frame_tokens, opt->max_head_dim)) != cudaSuccess)
     return cuda_fail(e, "no usable kernel image for this device (built for sm_103a)");
   if ((e = ipv::select_prepare(IPV_MAX_TOKENS)) != cudaSuccess) return cuda_fail(e, "select kernel set-up");
-  if ((e = ipv::pipeline_prepare()) != cudaSuccess) return cuda_fail(e, "pipeline kernel set-up");
+  if ((e = ipv::window_prepare()) != cudaSuccess) return cuda_fail(e, "fused kernel set-up");
   if ((e = ipv::pool_prepare()) != cudaSuccess) return cuda_fail(e, "pooling kernel set-up");
   State s;
   s.opt = *opt;
@@ -352,25 +404,25 @@ ipv_status ipv_init(const ipv_options* opt) {
   const size_t score_bytes = static_cast<size_t>(opt->max_slabs) * opt->token_capacity * sizeof(float);
   const size_t m_bytes =
       static_cast<size_t>(opt->max_slabs) * opt->max_frame_tokens * opt->max_head_dim * sizeof(float);
-  const size_t flag_bytes = ipv::kPipeFlags * static_cast<size_t>(opt->max_slabs) * sizeof(unsigned);
+  const size_t flag_bytes = ipv::kWinFlags * static_cast<size_t>(opt->max_slabs) * sizeof(unsigned);
   if (cudaMalloc(&s.tar, score_bytes) != cudaSuccess || cudaMalloc(&s.van, score_bytes) != cudaSuccess ||
       cudaMalloc(&s.m, m_bytes) != cudaSuccess ||
       (opt->van_pool && cudaMalloc(&s.pooled, score_bytes) != cudaSuccess) ||
       (opt->head_shared && (cudaMalloc(&s.kk, score_bytes) != cudaSuccess ||
                             cudaMalloc(&s.tar_l, score_bytes) != cudaSuccess ||
                             cudaMalloc(&s.van_l, score_bytes) != cudaSuccess)) ||
-      cudaMalloc(&s.pstate, sizeof(ipv::PipeState)) != cudaSuccess ||
-      cudaMalloc(&s.pflags, flag_bytes) != cudaSuccess || cudaMalloc(&s.claim, 3 * sizeof(unsigned)) != cudaSuccess) {
+      cudaMalloc(&s.wstate, sizeof(ipv::WinState)) != cudaSuccess ||
+      cudaMalloc(&s.wflags, flag_bytes) != cudaSuccess || cudaMalloc(&s.claim, 3 * sizeof(unsigned)) != cudaSuccess) {
     cudaGetLastError();
     free_scratch(s);
     return fail(IPV_ENOMEM, "scratch of %zu bytes could not be allocated",
                 (2 + opt->van_pool + 3 * opt->head_shared) * score_bytes + m_bytes);
   }
-  if ((e = cudaMemset(s.pstate, 0, sizeof(ipv::PipeState))) != cudaSuccess ||
-      (e = cudaMemset(s.pflags, 0, flag_bytes)) != cudaSuccess ||
+  if ((e = cudaMemset(s.wstate, 0, sizeof(ipv::WinState))) != cudaSuccess ||
+      (e = cudaMemset(s.wflags, 0, flag_bytes)) != cudaSuccess ||
       (e = cudaMemset(s.claim, 0, 3 * sizeof(unsigned))) != cudaSuccess) {
     free_scratch(s);
-    return cuda_fail(e, "clearing the pipeline state");
+    return cuda_fail(e, "clearing the fused pass's counters");
   }
   s.ready = true;
   g = s;
@@ -414,7 +466,6 @@ ipv_status ipv_score(const ipv_kv* k, const ipv_kv* v, int n_layers, int n_kv_he
   a.zero_recent = 1;
   a.van_recent = g.opt.van_pool;
   a.num_sms = g.num_sms;
-  a.error = &g.pstate->error;
   const bool tar_frame = g.opt.ablation == IPV_ABLATION_TAR_FRAME;
   if (tar_frame && k->patch_id[k->cur] && !k->frame_id[k->cur])
     return fail(IPV_EINVAL, "the frame-level TaR needs frame ids for a cache with patch ids");
@@ -529,7 +580,6 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   a.zero_recent = 0;
   a.van_recent = g.opt.van_pool;
   a.num_sms = g.num_sms;
-  a.error = &g.pstate->error;
 
   ipv::SelectArgs sa{};
   sa.tar = g.opt.head_shared ? g.tar_l : g.tar;
@@ -579,42 +629,28 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
     v->cur = 1 - v->cur;
     return IPV_OK;
   }
-  if (g.opt.single_kernel) {
-    if (g.pipe_dirty) {
-      if ((e = cudaMemsetAsync(g.pstate, 0, sizeof(ipv::PipeState), st)) != cudaSuccess ||
-          (e = cudaMemsetAsync(g.pflags, 0, ipv::kPipeFlags * sh.S * sizeof(unsigned), st)) != cudaSuccess)
-        return cuda_fail(e, "clearing the pipeline state");
-      g.pipe_dirty = false;
+  if (g.opt.single_kernel && !k->patch_id[k->cur]) {
+    // The fused pass scores a cache that has never been compacted (row n is
+    // patch n mod p); a cache with patch ids goes through the step kernels.
+    ipv::WinArgs wa{};
+    if (fused_args(a, sa, ga, sh, budget, &wa)) {
+      if (g.win_dirty) {
+        if ((e = cudaMemsetAsync(g.wstate, 0, offsetof(ipv::WinState, error), st)) != cudaSuccess ||
+            (e = cudaMemsetAsync(g.wflags, 0, ipv::kWinFlags * sh.S * sizeof(unsigned), st)) != cudaSuccess)
+          return cuda_fail(e, "clearing the fused pass's counters");
+        g.win_dirty = false;
+      }
+      prof_begin(4, st);
+      e = ipv::launch_window(wa, fused_smem(wa), st);
+      prof_end(4, st);
+      if (e != cudaSuccess) {
+        g.win_dirty = true;
+        return cuda_fail(e, "fused pass");
+      }
+      k->cur = 1 - k->cur;
+      v->cur = 1 - v->cur;
+      return IPV_OK;
     }
-    ipv::PipeArgs pa{};
-    pa.sc = a;
-    pa.se = sa;
-    pa.ga = ga;
-    pa.state = g.pstate;
-    pa.flags = g.pflags;
-    const int64_t n_past = sh.N - sh.rp;
-    pa.n_sc = static_cast<int>((n_past + 1023) / 1024);
-    pa.rows_sc = static_cast<int>((n_past + pa.n_sc - 1) / pa.n_sc);
-    pa.n_ga = static_cast<int>((budget + 1023) / 1024);
-    pa.rows_ga = static_cast<int>((budget + pa.n_ga - 1) / pa.n_ga);
-    pa.group = 4;
-    pa.lead = 2;
-    pa.n_groups = static_cast<int>((sh.S + pa.group - 1) / pa.group);
-    pa.spin_limit = g.wait_limit;
-    pa.nst = ipv::pipeline_stages(sh.p, sh.D, elem_bytes());
-    // The selection needs its keys in shared memory as well (one item at a time).
-    if (ipv::pipeline_smem_bytes(sh.N - sh.rp) > ipv::kBulkSmemMax)
-      return fail(IPV_EINVAL, "n_tokens %lld too large for the single-kernel pass", static_cast<long long>(sh.N));
-    prof_begin(4, st);
-    e = ipv::launch_pipeline(pa, g.num_sms, st);
-    prof_end(4, st);
-    if (e != cudaSuccess) {
-      g.pipe_dirty = true;
-      return cuda_fail(e, "single-kernel pass");
-    }
-    k->cur = 1 - k->cur;
-    v->cur = 1 - v->cur;
-    return IPV_OK;
   }
 
   // Overlap: the compaction copies the recent rows (always kept) while the
@@ -777,14 +813,14 @@ ipv_status ipv_device_error(uint32_t* err_out) {
   cudaSetDevice(g.opt.device);
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
-  ipv::PipeState ps;
-  if ((e = cudaMemcpy(&ps, g.pstate, sizeof ps, cudaMemcpyDeviceToHost)) != cudaSuccess)
-    return cuda_fail(e, "reading the pipeline state");
-  *err_out = ps.error;
-  if (ps.error != 0u) {
-    ps.error = 0u;
-    if ((e = cudaMemcpy(g.pstate, &ps, sizeof ps, cudaMemcpyHostToDevice)) != cudaSuccess)
-      return cuda_fail(e, "clearing the pipeline error");
+  ipv::WinState ws;
+  if ((e = cudaMemcpy(&ws, g.wstate, sizeof ws, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "reading the fused pass's state");
+  *err_out = ws.error;
+  if (ws.error != 0u) {
+    ws.error = 0u;
+    if ((e = cudaMemcpy(g.wstate, &ws, sizeof ws, cudaMemcpyHostToDevice)) != cudaSuccess)
+      return cuda_fail(e, "clearing the fused pass's error word");
   }
   return IPV_OK;
 }

@@ -8,7 +8,11 @@
 namespace ipv {
 
 constexpr float kNormEps = 1e-12f;   // cos(a,b) = a.b / (max|a|,eps)(max|b|,eps)
-constexpr int kSelectThreads = 1024;
+#ifndef IPV_SELECT_THREADS
+#define IPV_SELECT_THREADS 1024
+#endif
+constexpr int kSelectThreads = IPV_SELECT_THREADS;  // threads of the step path's selection block
+constexpr int kSelectRegE = 16;  // past tokens per thread when the selection keeps its keys in registers
 constexpr int kSelectBins = 2048;
 constexpr int64_t kMaxTokens = 49152;  // IPV_MAX_TOKENS: selection keys live in shared memory
 
@@ -79,10 +83,7 @@ cudaError_t launch(void (*kernel)(Params...), unsigned grid, unsigned block, siz
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
-// ---------------------------------------------------------------- bulk copies
-// 1-D bulk copies (cp.async.bulk, the TMA engine) from global into shared
-// memory, completed on an mbarrier that also counts the bytes. Addresses and
-// sizes are multiples of 16 bytes.
+// ---------------------------------------------------------------- asynchronous copies
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -103,52 +104,6 @@ __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(smem_dst)), "l"(gsrc) : "memory");
 }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-
-// Makes barrier initialisation visible to the bulk-copy (async) proxy.
-__device__ __forceinline__ void mbar_init_fence() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar))
-      : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t done;
-  asm volatile(
-      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
-      : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return done != 0u;
-}
-
-// Orders this thread's earlier generic-proxy shared-memory accesses before
-// its later bulk copies into shared memory.
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-// Bounded wait for a barrier phase; false if it did not complete in time.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (int it = 0; it < (1 << 22); ++it)
-    if (mbar_try_wait(bar, parity)) return true;
-  return false;
-}
 
 // Elements held by one 16-byte chunk, widened to fp32.
 template <typename T>
@@ -208,18 +163,9 @@ struct ScoreArgs {
   float* kk;                // scoring only: if set, write per-head partial sums instead of scores:
                             // tar <- k.m_q, kk <- |k|^2, van <- |v|^2 (NaN without a patch)
   int num_sms;
-  unsigned* error;          // device word: bit 2 set if a bulk-copy wait timed out
 };
 
 int row_shape(int D, int is_bf16);  // encoded (lanes per row, chunks per lane)
-// Bulk-copy-fed scoring: shape code (lanes per row * 10 + chunks per lane,
-// 324 for 32 lanes x 4), shared memory for the m table plus an nst-stage
-// ring, and the deepest ring (<= kMaxStages, >= 2) that fits (0: none).
-constexpr int kMaxStages = 4;
-constexpr size_t kBulkSmemMax = 226 * 1024;  // 227 KB per block, less room for static shared memory
-int bulk_shape(int D, int is_bf16);
-size_t bulk_smem_bytes(int p, int D, int elem, int nst, int threads);
-int bulk_stages(int p, int D, int elem, int threads);
 cudaError_t launch_recent_mean(const ScoreArgs& a, cudaStream_t st);
 cudaError_t launch_score(const ScoreArgs& a, cudaStream_t st);
 size_t score_smem_bytes(int p, int D);
@@ -325,34 +271,39 @@ cudaError_t launch_frame_mean(const FrameMeanArgs& a, cudaStream_t st);
 cudaError_t pool_prepare();
 cudaError_t launch_pool(const PoolArgs& a, cudaStream_t st, bool pdl);
 
-// Single-kernel pass (pipeline.cu). The queue state lives in library scratch,
-// is zero before a launch and is reset by the kernel's last block.
-struct PipeState {
-  unsigned main_head;  // next main-queue ticket
-  unsigned sel_low;    // slabs below have their selection taken
-  unsigned gat_low;    // slabs below have all gather chunks handed out
-  unsigned exited;     // blocks that have left
-  unsigned error;      // bit 0: a score item's wait timed out; bit 1: an idle wait timed out
-  unsigned pad[3];
+// Fused pass (window.cu): one cooperative persistent kernel, streaming
+// blocks and owner blocks. Its counters live in library scratch, are zero
+// before a launch and are reset by the kernel's last block.
+struct WinState {
+  unsigned head;      // next streaming ticket
+  unsigned sel_head;  // next slab for an owner block
+  unsigned exited;    // blocks that have left
+  unsigned error;     // bit 0: an owner gave up waiting for its slab's scores,
+                      // bit 1: a gather item gave up waiting for its selection
+  unsigned pad[4];
 };
-constexpr int kPipeFlags = 5;  // per-slab words: mean, scores, select claim, select done, gather ticket
+constexpr int kWinFlags = 2;  // per-slab words: score items done, selection done
+constexpr size_t kWinSmemMax = 112 * 1024;  // two blocks per SM
+constexpr int kWinBlock = 512;  // threads of a fused-pass block
+constexpr int kWinRegE = 18;    // past tokens per owner thread: the selection's keys stay in registers
 
-struct PipeArgs {
-  ScoreArgs sc;      // tar/van/m point at library scratch
+struct WinArgs {
+  ScoreArgs sc;      // k, v, tar, van: the source half and library score scratch
   SelectArgs se;
   GatherArgs ga;
-  PipeState* state;
-  unsigned* flags;   // [kPipeFlags][n_slabs]
-  int n_sc, rows_sc; // score chunks per slab, past rows per chunk
-  int n_ga, rows_ga; // gather chunks per slab, kept rows per chunk
-  int group, lead, n_groups;
-  int nst;           // bulk-copy stages for score chunks (0: 16-byte loads)
+  WinState* state;
+  unsigned* flags;   // [kWinFlags][n_slabs]
+  int n_si;          // score items per slab (patch ranges)
+  int qmax;          // most patches in one score item
+  int n_gi, rows_gi; // gather items per slab, selected rows per gather item
+  int lag;           // slabs between a slab's score items and its gather items
+  int n_stream, n_owner;  // blocks of each kind
   int64_t spin_limit;
 };
 
-size_t pipeline_smem_bytes(int64_t n_past);
-int pipeline_stages(int p, int D, int elem);  // bulk-copy stages that fit (0: none)
-cudaError_t pipeline_prepare();
-cudaError_t launch_pipeline(const PipeArgs& a, int num_sms, cudaStream_t st);
+size_t window_smem_bytes(int qmax, int D, int elem, int r, int64_t n_past);
+cudaError_t window_prepare();
+cudaError_t window_blocks_per_sm(const WinArgs& a, size_t smem, int* per_sm);
+cudaError_t launch_window(const WinArgs& a, size_t smem, cudaStream_t st);
 
 }  // namespace ipv

@@ -15,7 +15,9 @@
 // On the first call on a device (the current device), the entry point sets
 // up that device once: it sets the kernels' shared-memory limits and looks up
 // the array's device address with cudaGetSymbolAddress. Make that first call
-// before any stream capture. All calls on a device share the one array, which
+// before any stream capture. The set-up is kept for the life of the process:
+// a cudaDeviceReset of that device after its first call is not supported.
+// All calls on a device share the one array, which
 // keeps whatever the previous call left: calls that may overlap on the GPU
 // (different streams, or different host threads) race on it and must be
 // ordered by the caller. Nothing in the array needs clearing between calls,
@@ -149,6 +151,16 @@ extern "C" ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype,
   const int64_t rp = static_cast<int64_t>(r) * p;
 
   // Working memory: TaR and VaN [S][n_tokens], m [S][p][head_dim] (fp32).
+  // The slab count is bounded by division first, so that the byte counts
+  // below cannot wrap around for any argument values.
+  if (S > INT32_MAX) return reject(IPV_EINVAL, "n_layers*n_kv_heads exceeds 2^31 - 1");
+  const uint64_t per_slab = 8u * static_cast<uint64_t>(n_tokens) + 4u * static_cast<uint64_t>(p) * head_dim;
+  if (evict && static_cast<uint64_t>(S) > IPV_STATIC_SCRATCH_BYTES / per_slab)
+    return reject(IPV_EINVAL,
+                  "this pass needs more than the %u bytes of working memory of ipv_compress_static "
+                  "(%lld slabs of %llu bytes; use ipv_compress, or fewer slabs per call)",
+                  static_cast<unsigned>(IPV_STATIC_SCRATCH_BYTES), static_cast<long long>(S),
+                  static_cast<unsigned long long>(per_slab));
   const size_t score_bytes = round256(static_cast<size_t>(S) * n_tokens * sizeof(float));
   const size_t m_bytes = round256(static_cast<size_t>(S) * p * head_dim * sizeof(float));
   if (evict && 2 * score_bytes + m_bytes > IPV_STATIC_SCRATCH_BYTES)
@@ -190,7 +202,6 @@ extern "C" ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype,
   a.van = van;
   a.zero_recent = 0;
   a.num_sms = dev->num_sms;
-  a.error = nullptr;
   if ((e = ipv::launch_recent_mean(a, cs)) != cudaSuccess) return cuda_reject(e, "recent-frame mean kernel");
   if ((e = ipv::launch_score(a, cs)) != cudaSuccess) return cuda_reject(e, "scoring kernel");
 

@@ -1,6 +1,6 @@
-// Device building blocks of the compression pass, shared by the staged
-// kernels (score.cu, select.cu, gather.cu) and the single-kernel pipeline
-// (pipeline.cu), so that both paths run exactly the same arithmetic.
+// Device building blocks of the compression pass, shared by the step kernels
+// (score.cu, select.cu, gather.cu) and the fused pass (window.cu), so that
+// both paths run exactly the same arithmetic.
 #pragma once
 
 #include "ipv_common.cuh"
@@ -158,6 +158,47 @@ __device__ __forceinline__ float4 load_m4(const float* p) {
   return *reinterpret_cast<const float4*>(p);  // written earlier in the same kernel
 }
 
+// The three sums of one row, reduced over its LPR lanes: k.m_q, |k|^2 and
+// |v|^2 (fp32, packed FMA per lane in chunk order, then a shuffle tree). kr
+// and vr hold the lane's CPL chunks of the K and V row; mq is the row's m_q.
+// Every scoring path uses this function, so all give the same bits.
+template <typename T, int LPR, int CPL, int MSRC>
+__device__ __forceinline__ void row_sums(const uint4* kr, const uint4* vr, const float* mq, int sub,
+                                         int n_chunks, float* dot, float* kk, float* vv) {
+  constexpr int E = Chunk<T>::kElems;
+  constexpr int P2 = Chunk<T>::kPairs;
+  float2 dot2 = make_float2(0.0f, 0.0f), kk2 = dot2, vv2 = dot2;
+#pragma unroll
+  for (int i = 0; i < CPL; ++i) {
+    const int c = sub + LPR * i;
+    float2 kx[P2], vx[P2];
+    Chunk<T>::widen2(kr[i], kx);
+    Chunk<T>::widen2(vr[i], vx);
+    if (c < n_chunks) {
+#pragma unroll
+      for (int e = 0; e < P2; e += 2) {
+        const float4 mv = load_m4<MSRC>(mq + c * E + 2 * e);
+        dot2 = fma2(kx[e], make_float2(mv.x, mv.y), dot2);
+        dot2 = fma2(kx[e + 1], make_float2(mv.z, mv.w), dot2);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < P2; ++e) {
+      kk2 = fma2(kx[e], kx[e], kk2);
+      vv2 = fma2(vx[e], vx[e], vv2);
+    }
+  }
+  *dot = group_sum<LPR>(dot2.x + dot2.y);
+  *kk = group_sum<LPR>(kk2.x + kk2.y);
+  *vv = group_sum<LPR>(vv2.x + vv2.y);
+}
+
+// Sec. 3.1 Eq. (tar) and Sec. 3.2 from a row's sums: s_TaR = -(k . m_q) /
+// max(|k|, eps), with max(|k|, eps) = sqrt(max(|k|^2, eps^2)); s_VaN = |v|.
+__device__ __forceinline__ float tar_of(float dot, float kk) {
+  return -dot * rsqrtf(fmaxf(kk, kNormEps * kNormEps));
+}
+
 // TaR and VaN of past rows [lo, hi) of slab s by every warp of the block
 // (block-uniform arguments). Sec. 3.1 Eq. (tar): s_TaR = -(k . m_q) / max(|k|, eps);
 // Sec. 3.2: s_VaN = |v|. Each warp step covers 32/LPR consecutive rows; kU
@@ -165,8 +206,6 @@ __device__ __forceinline__ float4 load_m4(const float* p) {
 template <typename T, int LPR, int CPL, int kU, int MSRC>
 __device__ __forceinline__ void score_segment(const ScoreArgs& a, int64_t s, int lo, int hi,
                                               const float* mtab, int ms) {
-  constexpr int E = Chunk<T>::kElems;
-  constexpr int P2 = Chunk<T>::kPairs;
   constexpr int RPW = 32 / LPR;
   const int lane = threadIdx.x & 31;
   const int sub = lane % LPR, grp = lane / LPR;
@@ -214,40 +253,17 @@ __device__ __forceinline__ void score_segment(const ScoreArgs& a, int64_t s, int
       const int n = base + off[u];
       const bool q_ok = q[u] < p;
       const float* mq = mtab + static_cast<int64_t>(q_ok ? q[u] : 0) * ms;
-      float2 dot2 = make_float2(0.0f, 0.0f), kk2 = dot2, vv2 = dot2;
-#pragma unroll
-      for (int i = 0; i < CPL; ++i) {
-        const int c = sub + LPR * i;
-        float2 kx[P2], vx[P2];
-        Chunk<T>::widen2(kr[u][i], kx);
-        Chunk<T>::widen2(vr[u][i], vx);
-        if (c < n_chunks) {
-#pragma unroll
-          for (int e = 0; e < P2; e += 2) {
-            const float4 mv = load_m4<MSRC>(mq + c * E + 2 * e);
-            dot2 = fma2(kx[e], make_float2(mv.x, mv.y), dot2);
-            dot2 = fma2(kx[e + 1], make_float2(mv.z, mv.w), dot2);
-          }
-        }
-#pragma unroll
-        for (int e = 0; e < P2; ++e) {
-          kk2 = fma2(kx[e], kx[e], kk2);
-          vv2 = fma2(vx[e], vx[e], vv2);
-        }
-      }
-      const float dot = group_sum<LPR>(dot2.x + dot2.y);
-      const float kk = group_sum<LPR>(kk2.x + kk2.y);
-      const float vv = group_sum<LPR>(vv2.x + vv2.y);
+      float dot, kk, vv;
+      row_sums<T, LPR, CPL, MSRC>(kr[u], vr[u], mq, sub, n_chunks, &dot, &kk, &vv);
       if (sub == 0 && n < hi) {
-        // max(|k|, eps) = sqrt(max(|k|^2, eps^2)). A patch id outside [0, p)
-        // has no recent-frame partner: NaN scores rank below every number,
-        // so such a token is never preferred.
+        // A patch id outside [0, p) has no recent-frame partner: NaN scores
+        // rank below every number, so such a token is never preferred.
         if (a.kk) {  // the shared index set: this head's partial sums
           tar[n] = q_ok ? dot : __int_as_float(0x7fc00000);
           a.kk[s * a.n_tokens + n] = kk;
           van[n] = q_ok ? vv : __int_as_float(0x7fc00000);
         } else {
-          tar[n] = q_ok ? -dot * rsqrtf(fmaxf(kk, kNormEps * kNormEps)) : __int_as_float(0x7fc00000);
+          tar[n] = q_ok ? tar_of(dot, kk) : __int_as_float(0x7fc00000);
           van[n] = q_ok ? sqrtf(vv) : __int_as_float(0x7fc00000);
         }
       }
@@ -257,151 +273,45 @@ __device__ __forceinline__ void score_segment(const ScoreArgs& a, int64_t s, int
   }
 }
 
-// Shared-memory bookkeeping of the bulk-copy ring (static, per block).
-struct BulkRing {
-  uint64_t full[kMaxStages];    // completes when a stage's copies have landed
-  unsigned done[kMaxStages];    // warps finished with the stage's current chunk
-  unsigned issued[kMaxStages];  // copies ever issued into the stage
-};
-
-__device__ __forceinline__ void ring_init(BulkRing& rg, int nst) {  // thread 0
-  for (int i = 0; i < nst; ++i) {
-    mbar_init(&rg.full[i], 1u);
-    rg.done[i] = 0u;
-    rg.issued[i] = 0u;
-  }
-  mbar_init_fence();
-}
-
-// Copies a slab's m table ([p][D] fp32, global) into shared memory in the
-// layout score_segment_bulk reads: each row split into E/4 planes, plane j
-// holding floats 4j..4j+3 of every 16-byte chunk of K (E elements per chunk),
-// so the lanes of a row read 16 consecutive bytes each. RO: the table is not
-// written by the running kernel (read through the non-coherent path).
-template <typename T, bool RO>
-__device__ __forceinline__ void load_m_planes(const float* m_slab, float* m_tab, int p, int D) {
-  constexpr int kPlanes = Chunk<T>::kElems / 4;
-  const int d4 = D / 4;  // float4s per row
-  const float4* src = reinterpret_cast<const float4*>(m_slab);
-  float4* dst = reinterpret_cast<float4*>(m_tab);
-  for (int i = threadIdx.x; i < p * d4; i += blockDim.x) {
-    const int q = i / d4, f = i - q * d4;
-    const int c = f / kPlanes, pl = f - c * kPlanes;
-    dst[q * d4 + pl * (d4 / kPlanes) + c] = RO ? __ldg(src + i) : src[i];
-  }
-}
-
-// Bulk-copy-fed version of score_segment. A ring of nst stages, each R
-// consecutive rows of K followed by the same rows of V (R = all warps' rows of
-// one warp step, 16 KB per copy at the usual shapes), is filled by cp.async.bulk.
-// Warps consume every stage independently and count themselves out; the warp
-// that finishes a stage last refills it with the chunk nst steps ahead, so no
-// block-wide barrier is taken while streaming and copies stay large. 8/16/32
-// lanes share a row: a shared-memory phase reads one row's 128 contiguous
-// bytes (no bank conflicts). m_tab is the slab's m table in shared memory in
-// the layout of load_m_planes; seq counts the stages this block has used (barrier parity) and is
-// kept by the caller across segments. On a barrier timeout the warp stops,
-// sets bit 2 of *a.error, and the block drains its copies before returning.
+// TaR and VaN of the past rows of patches [q0, q0 + nq) of slab s, for a
+// cache that has never been compacted (row n = f p + q; f < f_past) by every
+// warp of the block. mtab holds m_q of those patches, row q - q0 at
+// (q - q0) * ms floats (shared memory). Same arithmetic as score_segment.
 template <typename T, int LPR, int CPL>
-__device__ __forceinline__ void score_segment_bulk(const ScoreArgs& a, int64_t s, int lo, int hi,
-                                                   const float* m_tab, char* stages, int nst,
-                                                   BulkRing& rg, uint32_t& seq) {
-  constexpr int P2 = Chunk<T>::kPairs;
-  constexpr int kPlanes = Chunk<T>::kElems / 4;
+__device__ __forceinline__ void score_patch_rows(const ScoreArgs& a, int64_t s, int q0, int nq, int f_past,
+                                                 const float* mtab, int ms) {
   constexpr int RPW = 32 / LPR;
   const int lane = threadIdx.x & 31;
   const int sub = lane % LPR, grp = lane / LPR;
   const int warp = threadIdx.x >> 5, n_warps = blockDim.x >> 5;
   const int row_bytes = a.D * static_cast<int>(sizeof(T));
   const int n_chunks = row_bytes / 16;
-  const int R = n_warps * RPW;
-  const int stage_bytes = 2 * R * row_bytes;
-  const int p = a.p;
+  const int n_rows = f_past * nq;
+  const int G = n_warps * RPW;
   const char* kslab = static_cast<const char*>(a.k) + s * a.cap * row_bytes;
   const char* vslab = static_cast<const char*>(a.v) + s * a.cap * row_bytes;
-  const uint16_t* pid = a.patch_id ? a.patch_id + s * a.cap : nullptr;
   float* tar = a.tar + s * a.n_tokens;
   float* van = a.van + s * a.n_tokens;
-  const int n_steps = (hi - lo + R - 1) / R;
-  const int my_row = warp * RPW + grp;
-  const uint32_t seq0 = seq;
-
-  auto issue = [&](int j) {  // one thread
-    const uint32_t slot = (seq0 + j) % nst;
-    const int r0 = lo + j * R;
-    const uint32_t bytes = static_cast<uint32_t>(min(R, hi - r0) * row_bytes);
-    char* dst = stages + slot * stage_bytes;
-    fence_proxy_async_smem();  // earlier ordinary accesses to this stage come first
-    rg.issued[slot] += 1u;
-    mbar_expect_tx(&rg.full[slot], 2u * bytes);
-    bulk_g2s(dst, kslab + static_cast<int64_t>(r0) * row_bytes, bytes, &rg.full[slot]);
-    bulk_g2s(dst + R * row_bytes, vslab + static_cast<int64_t>(r0) * row_bytes, bytes, &rg.full[slot]);
-  };
-  if (threadIdx.x == 0)
-    for (int j = 0; j < nst && j < n_steps; ++j) issue(j);
-
-  int j = 0;
-  for (; j < n_steps; ++j) {
-    const uint32_t slot = (seq0 + j) % nst;
-    const bool landed = mbar_wait(&rg.full[slot], ((seq0 + j) / nst) & 1u);
-    if (__any_sync(0xffffffffu, !landed)) break;
-    const char* kst = stages + slot * stage_bytes + my_row * row_bytes;
-    const char* vst = kst + R * row_bytes;
-    const int n = lo + j * R + my_row;
-    const bool ok = n < hi;
-    const int q = pid ? (ok ? static_cast<int>(pid[n]) : 0) : n % p;
-    const bool q_ok = q < p;
-    const float* mq = m_tab + (q_ok ? q : 0) * a.D;
-    float2 dot2 = make_float2(0.0f, 0.0f), kk2 = dot2, vv2 = dot2;
+  for (int base = 0; base < n_rows; base += G) {  // warp-uniform
+    const int i = base + warp * RPW + grp;
+    const bool ok = i < n_rows;
+    const int f = ok ? i / nq : 0;
+    const int qi = ok ? i - f * nq : 0;
+    const int64_t n = static_cast<int64_t>(f) * a.p + q0 + qi;
+    uint4 kr[CPL], vr[CPL];
 #pragma unroll
-    for (int k = 0; k < CPL; ++k) {
-      const int c = sub + LPR * k;
-      if (ok && c < n_chunks) {
-        float2 kx[P2], vx[P2];
-        Chunk<T>::widen2(*reinterpret_cast<const uint4*>(kst + c * 16), kx);
-        Chunk<T>::widen2(*reinterpret_cast<const uint4*>(vst + c * 16), vx);
-#pragma unroll
-        for (int e = 0; e < P2; e += 2) {
-          // m_tab row layout: plane e/2 holds floats 2e..2e+3 of every chunk.
-          const float4 mv = *reinterpret_cast<const float4*>(mq + (e / 2) * (a.D / kPlanes) + c * 4);
-          dot2 = fma2(kx[e], make_float2(mv.x, mv.y), dot2);
-          dot2 = fma2(kx[e + 1], make_float2(mv.z, mv.w), dot2);
-        }
-#pragma unroll
-        for (int e = 0; e < P2; ++e) {
-          kk2 = fma2(kx[e], kx[e], kk2);
-          vv2 = fma2(vx[e], vx[e], vv2);
-        }
-      }
+    for (int c = 0; c < CPL; ++c) {
+      const int ch = sub + LPR * c;
+      const bool ld = ok && ch < n_chunks;
+      kr[c] = ld ? ld_stream(kslab + n * row_bytes + ch * 16) : make_uint4(0, 0, 0, 0);
+      vr[c] = ld ? ld_stream(vslab + n * row_bytes + ch * 16) : make_uint4(0, 0, 0, 0);
     }
-    const float dot = group_sum<LPR>(dot2.x + dot2.y);
-    const float kk = group_sum<LPR>(kk2.x + kk2.y);
-    const float vv = group_sum<LPR>(vv2.x + vv2.y);
+    float dot, kk, vv;
+    row_sums<T, LPR, CPL, kMSmem>(kr, vr, mtab + qi * ms, sub, n_chunks, &dot, &kk, &vv);
     if (sub == 0 && ok) {
-      // max(|k|, eps) = sqrt(max(|k|^2, eps^2)). A patch id outside [0, p)
-      // has no recent-frame partner: NaN scores rank below every number.
-      tar[n] = q_ok ? -dot * rsqrtf(fmaxf(kk, kNormEps * kNormEps)) : __int_as_float(0x7fc00000);
-      van[n] = q_ok ? sqrtf(vv) : __int_as_float(0x7fc00000);
+      tar[n] = tar_of(dot, kk);
+      van[n] = sqrtf(vv);
     }
-    __syncwarp();
-    if (lane == 0) {
-      __threadfence_block();  // this warp's reads of the stage are done
-      if (atomicAdd(&rg.done[slot], 1u) == static_cast<unsigned>(n_warps - 1)) {
-        rg.done[slot] = 0u;  // last warp out: refill the stage
-        __threadfence_block();
-        if (j + nst < n_steps) issue(j + nst);
-      }
-    }
-  }
-  seq = seq0 + n_steps;
-  if (__syncthreads_or(j < n_steps)) {  // a barrier timed out somewhere
-    if (threadIdx.x == 0) {
-      atomicOr(a.error, 4u);
-      for (int k = 0; k < nst; ++k)  // wait for the last copy issued into each stage
-        if (rg.issued[k]) mbar_wait(&rg.full[k], (rg.issued[k] - 1u) & 1u);
-      for (int k = 0; k < nst; ++k) rg.done[k] = 0u;
-    }
-    __syncthreads();
   }
 }
 
@@ -412,13 +322,19 @@ __device__ __forceinline__ void score_segment_bulk(const ScoreArgs& a, int64_t s
 // before its final TopK). Ties go to the lower index; NaN ranks lowest.
 //
 // One block of NT threads per slab; scores live in shared memory as
-// order-preserving uint32 keys. A stage finds its k winners without a sort: a
-// 2048-bin histogram linear in the score value over [min, max] of the
-// candidates (a monotone map, so every bin above the one holding the k-th
-// winner is taken whole); the candidates of that boundary bin are ranked
-// exactly against each other with the index tie-break. A boundary bin of
-// more than NT candidates falls back to an exact search over integer key
-// windows with ties counted by a block-wide prefix sum in index order.
+// order-preserving uint32 keys. A stage finds its k winners without a sort,
+// from a 2048-bin histogram whose bins are a monotone map of the score (so
+// every bin above the one holding the k-th winner is taken whole):
+//   TaR, a mean of cosines in [-1, 1]: 2048 equal bins over [-1, 1], values
+//        outside folded into the end bins, so that its histogram is built in
+//        the pass that loads the scores;
+//   VaN: 2048 equal bins over [min, max] of every past token's VaN, a range
+//        taken in that same pass (the VaN stage's candidates are a subset).
+// The candidates of the boundary bin are ranked exactly against each other
+// with the index tie-break. A boundary bin of more than NT candidates falls
+// back to an exact search over integer key windows with ties counted by a
+// block-wide prefix sum in index order. Any score values are handled
+// exactly; the bins only decide how much work the exact steps have.
 constexpr uint32_t kTaken = 0xFFFFFFFFu;  // VaN pick (never a score key)
 constexpr uint32_t kExcluded = 0u;        // TaR pick, excluded from the VaN stage
 constexpr uint32_t kNanKey = 1u;          // score_key of every NaN
@@ -434,11 +350,12 @@ struct SelShared {
   uint32_t list_n;
 };
 
-// Shared memory of select_slab: keys[pad4(n_past)], hist[2048], list_key[NT],
-// list_idx[NT], and with a.van_smem the VaN scores[pad4(n_past)].
+// Shared memory of select_slab: keys[pad4(n_past)], hist_tar[2048],
+// hist_van[2048], list_key[NT], list_idx[NT], and with a.van_smem the VaN
+// scores[pad4(n_past)].
 template <int NT>
 __host__ __device__ constexpr size_t select_smem_words(int64_t n_past, bool van_smem = false) {
-  return static_cast<size_t>((n_past + 3) & ~3LL) * (van_smem ? 2 : 1) + kSelectBins + 2 * NT;
+  return static_cast<size_t>((n_past + 3) & ~3LL) * (van_smem ? 2 : 1) + 2 * kSelectBins + 2 * NT;
 }
 
 __device__ __forceinline__ bool is_cand(uint32_t k) { return k != kExcluded && k != kTaken; }
@@ -447,9 +364,19 @@ __device__ __forceinline__ float key_value(uint32_t k) {  // inverse of score_ke
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
 }
 
-__device__ __forceinline__ int value_bin(float v, float vmin, float scale) {  // monotone
-  const int b = static_cast<int>((v - vmin) * scale);
-  return b < kSelectBins - 1 ? b : kSelectBins - 1;
+// A monotone non-decreasing map of a score (not NaN) to one of 2048 bins:
+// floor((v - lo) * scale), folded into [0, 2047] (scale 0: every value in bin 0).
+struct Bins {
+  float lo, scale;
+  __device__ __forceinline__ int of(float v) const {
+    return static_cast<int>(fminf(fmaxf((v - lo) * scale, 0.0f), 2047.0f));
+  }
+};
+__device__ __forceinline__ Bins tar_bins() { return Bins{-1.0f, 1024.0f}; }
+__device__ __forceinline__ Bins range_bins(float vmin, float vmax) {
+  const float range = vmax - vmin;
+  const float scale = static_cast<float>(kSelectBins) / range;
+  return Bins{vmin, (range > 0.0f && scale < INFINITY) ? scale : 0.0f};
 }
 
 __device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v) {
@@ -481,6 +408,56 @@ __device__ uint32_t block_excl_scan(uint32_t v, uint32_t* total, SelShared& sh) 
   *total = sh.bcast[7];
   __syncthreads();
   return out;
+}
+
+// Block-wide sum of v (every thread gets it).
+template <int NT>
+__device__ uint32_t block_sum(uint32_t v, SelShared& sh) {
+  uint32_t tot;
+  block_excl_scan<NT>(v, &tot, sh);
+  return tot;
+}
+
+// Block-wide sum of *cnt, min of *lo and max of *hi (every thread gets them).
+template <int NT>
+__device__ void block_reduce3(uint32_t* cnt, float* lo, float* hi, SelShared& sh) {
+  constexpr int W = NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t c = *cnt;
+  float l = *lo, h = *hi;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    c += __shfl_xor_sync(0xffffffffu, c, off);
+    l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
+    h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
+  }
+  if (lane == 0) {
+    sh.warp_a[warp] = c;
+    sh.warp_f[warp] = l;
+    sh.warp_g[warp] = h;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    c = lane < W ? sh.warp_a[lane] : 0u;
+    l = lane < W ? sh.warp_f[lane] : INFINITY;
+    h = lane < W ? sh.warp_g[lane] : -INFINITY;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      c += __shfl_xor_sync(0xffffffffu, c, off);
+      l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
+      h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
+    }
+    if (lane == 0) {
+      sh.bcast[5] = c;
+      sh.fcast[0] = l;
+      sh.fcast[1] = h;
+    }
+  }
+  __syncthreads();
+  *cnt = sh.bcast[5];
+  *lo = sh.fcast[0];
+  *hi = sh.fcast[1];
+  __syncthreads();
 }
 
 template <int NT>
@@ -515,58 +492,6 @@ __device__ void block_minmax(uint32_t lo, uint32_t hi, uint32_t* out_lo, uint32_
   *out_lo = sh.bcast[0];
   *out_hi = sh.bcast[1];
   __syncthreads();
-}
-
-struct Stats {  // value range and NaN count of a stage's candidates
-  float vmin, vmax;
-  uint32_t n_nan;
-};
-
-__device__ __forceinline__ void stats_add(Stats& st, float v) {
-  if (v != v) {
-    ++st.n_nan;
-  } else {
-    st.vmin = fminf(st.vmin, v);
-    st.vmax = fmaxf(st.vmax, v);
-  }
-}
-
-template <int NT>
-__device__ Stats block_stats(Stats st, SelShared& sh) {
-  constexpr int W = NT / 32;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    st.vmin = fminf(st.vmin, __shfl_xor_sync(0xffffffffu, st.vmin, off));
-    st.vmax = fmaxf(st.vmax, __shfl_xor_sync(0xffffffffu, st.vmax, off));
-    st.n_nan += __shfl_xor_sync(0xffffffffu, st.n_nan, off);
-  }
-  if (lane == 0) {
-    sh.warp_f[warp] = st.vmin;
-    sh.warp_g[warp] = st.vmax;
-    sh.warp_a[warp] = st.n_nan;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    st.vmin = lane < W ? sh.warp_f[lane] : INFINITY;
-    st.vmax = lane < W ? sh.warp_g[lane] : -INFINITY;
-    st.n_nan = lane < W ? sh.warp_a[lane] : 0u;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      st.vmin = fminf(st.vmin, __shfl_xor_sync(0xffffffffu, st.vmin, off));
-      st.vmax = fmaxf(st.vmax, __shfl_xor_sync(0xffffffffu, st.vmax, off));
-      st.n_nan += __shfl_xor_sync(0xffffffffu, st.n_nan, off);
-    }
-    if (lane == 0) {
-      sh.fcast[0] = st.vmin;
-      sh.fcast[1] = st.vmax;
-      sh.bcast[0] = st.n_nan;
-    }
-  }
-  __syncthreads();
-  Stats out{sh.fcast[0], sh.fcast[1], sh.bcast[0]};
-  __syncthreads();
-  return out;
 }
 
 // The bin holding the k-th largest candidate (bins scanned from the top;
@@ -607,8 +532,9 @@ __device__ void boundary_bin(const uint32_t* hist, uint32_t k, SelShared& sh, ui
 // holding cnt candidates of which the k largest are wanted (all candidates
 // above hi are taken already). Winners: candidates with key > *T plus the
 // *take_eq lowest-index ones with key == *T; *cnt_eq counts those equal to *T.
-// The window shrinks at least 2048-fold per round (4 rounds for 32-bit
-// keys); the hard round limit only guards against a broken invariant.
+// hist is scratch. The window shrinks at least 2048-fold per round (4 rounds
+// for 32-bit keys); the hard round limit only guards against a broken
+// invariant.
 template <int NT>
 __device__ void window_search(const uint32_t* key, int n, uint32_t lo, uint32_t hi, uint32_t k,
                               uint32_t cnt, uint32_t* hist, SelShared& sh, uint32_t* T,
@@ -618,10 +544,11 @@ __device__ void window_search(const uint32_t* key, int n, uint32_t lo, uint32_t 
     const uint64_t W = static_cast<uint64_t>(hi - lo) + 1u;
     for (int b = threadIdx.x; b < kSelectBins; b += NT) hist[b] = 0u;
     __syncthreads();
-    for (int i = threadIdx.x; i < n; i += NT) {
-      const uint32_t x = key[i];
-      if (x >= lo && x <= hi)
-        atomicAdd(&hist[(static_cast<uint64_t>(x - lo) * kSelectBins) / W], 1u);
+    for (int i0 = threadIdx.x & ~31; i0 < n; i0 += NT) {  // warp-uniform
+      const int i = i0 + (threadIdx.x & 31);
+      const uint32_t x = i < n ? key[i] : kExcluded;
+      const bool in = i < n && x >= lo && x <= hi;
+      if (in) atomicAdd(&hist[(static_cast<uint64_t>(x - lo) * kSelectBins) / W], 1u);
     }
     __syncthreads();
     uint32_t bsel, above, cnt_b;
@@ -649,111 +576,103 @@ __device__ void window_search(const uint32_t* key, int n, uint32_t lo, uint32_t 
 
 // How a stage's winners are recognised in the marking pass (block-uniform).
 struct Plan {
-  int mode;  // 0 none, 1 every candidate, 2 key threshold, 3 value bin (+ pre-marked)
+  int mode;  // 0 none, 1 every candidate, 2 key threshold, 3 bin threshold (+ pre-marked)
+  Bins bins;
   uint32_t T, take, cnt_eq;
   int bthr;
-  float vmin, scale;
 };
 
-// Decides a stage taking the k best of n_cand candidates. Boundary-bin
-// winners found by direct ranking are marked in place with `mark`.
+// Decides a stage taking the k best of n_cand candidates (n_nan of them NaN);
+// hist holds the candidates' numbers in the stage's bins. Boundary-bin
+// winners found by direct ranking are marked in place with `mark`. scratch
+// (2048 words) may be overwritten.
 template <int NT>
-__device__ Plan plan_stage(uint32_t* key, int n, uint32_t k, uint32_t n_cand, Stats st,
-                           uint32_t mark, uint32_t* hist, uint32_t* list_key, uint32_t* list_idx,
-                           SelShared& sh) {
+__device__ Plan plan_stage(uint32_t* key, int n, uint32_t k, uint32_t n_cand, uint32_t n_nan, Bins bins,
+                           const uint32_t* hist, uint32_t* scratch, uint32_t mark, uint32_t* list_key,
+                           uint32_t* list_idx, SelShared& sh) {
   Plan P{};
+  P.bins = bins;
   if (k == 0u) return P;
   if (k >= n_cand) {
     P.mode = 1;
     return P;
   }
-  const uint32_t n_num = n_cand - st.n_nan;
+  const uint32_t n_num = n_cand - n_nan;
   P.mode = 2;
   if (k > n_num) {  // every number, then the lowest-index NaNs
     P.T = kNanKey;
     P.take = k - n_num;
-    P.cnt_eq = st.n_nan;
+    P.cnt_eq = n_nan;
     return P;
   }
-  if (st.vmin == st.vmax) {  // all numbers equal
-    P.T = score_key(st.vmin);
-    P.take = k;
-    P.cnt_eq = n_num;
-    return P;
-  }
-  const float range = st.vmax - st.vmin;
-  const float scale = static_cast<float>(kSelectBins) / range;
-  uint32_t lo = score_key(st.vmin), hi = score_key(st.vmax), k_rem = k, cnt = n_num;
-  if (range < INFINITY && scale < INFINITY) {
-    for (int b = threadIdx.x; b < kSelectBins; b += NT) hist[b] = 0u;
+  uint32_t bsel, above, cnt_b;
+  boundary_bin<NT>(hist, k, sh, &bsel, &above, &cnt_b);
+  uint32_t lo = 2u, hi = kTaken - 1u, k_rem = k, cnt = n_num;
+  if (bsel != kNoBin) {  // always: the histogram holds n_num >= k numbers
+    k_rem = k - above;
+    P.mode = 3;
+    if (cnt_b == k_rem) {  // the whole boundary bin is taken
+      P.bthr = static_cast<int>(bsel) - 1;
+      return P;
+    }
+    P.bthr = static_cast<int>(bsel);
+    const int lane = threadIdx.x & 31;
     if (threadIdx.x == 0) sh.list_n = 0u;
     __syncthreads();
+    if (cnt_b <= static_cast<uint32_t>(NT)) {
+      // Collect the boundary bin's candidates (a ballot per warp, one atomic).
+      for (int i0 = threadIdx.x - lane; i0 < n; i0 += NT) {  // warp-uniform
+        const int i = i0 + lane;
+        const uint32_t x = i < n ? key[i] : kExcluded;
+        const bool in = is_cand(x) && x != kNanKey && bins.of(key_value(x)) == static_cast<int>(bsel);
+        const unsigned m = __ballot_sync(0xffffffffu, in);
+        if (m == 0u) continue;
+        uint32_t base = 0u;
+        if (lane == __ffs(m) - 1) base = atomicAdd(&sh.list_n, static_cast<uint32_t>(__popc(m)));
+        base = __shfl_sync(0xffffffffu, base, __ffs(m) - 1);
+        if (in) {
+          const uint32_t j = base + __popc(m & ((1u << lane) - 1u));
+          if (j < static_cast<uint32_t>(NT)) {
+            list_key[j] = x;
+            list_idx[j] = static_cast<uint32_t>(i);
+          }
+        }
+      }
+      __syncthreads();
+      const uint32_t m = min(sh.list_n, static_cast<uint32_t>(NT));
+      // T threads rank one candidate (T m <= NT, T <= 32, aligned within a
+      // warp), each against every T-th other one, then sum over the T lanes.
+      uint32_t T = 32u;
+      while (T > 1u && T * m > static_cast<uint32_t>(NT)) T >>= 1;
+      const uint32_t cand = threadIdx.x / T, sub = threadIdx.x % T;
+      uint32_t rank = 0u, kt = 0u, it = 0u;
+      if (cand < m) {
+        kt = list_key[cand];
+        it = list_idx[cand];
+        for (uint32_t j = sub; j < m; j += T) {
+          const uint32_t kj = list_key[j];
+          rank += (kj > kt || (kj == kt && list_idx[j] < it)) ? 1u : 0u;
+        }
+      }
+      for (uint32_t off = T >> 1; off > 0u; off >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off);
+      if (cand < m && sub == 0u && rank < k_rem) key[it] = mark;
+      __syncthreads();
+      return P;
+    }
+    // Too many candidates in the bin: exact search inside its key range.
+    uint32_t blo = 0xFFFFFFFFu, bhi = 0u;
     for (int i = threadIdx.x; i < n; i += NT) {
       const uint32_t x = key[i];
-      if (is_cand(x) && x != kNanKey) atomicAdd(&hist[value_bin(key_value(x), st.vmin, scale)], 1u);
+      if (is_cand(x) && x != kNanKey && bins.of(key_value(x)) == static_cast<int>(bsel)) {
+        blo = min(blo, x);
+        bhi = max(bhi, x);
+      }
     }
-    __syncthreads();
-    uint32_t bsel, above, cnt_b;
-    boundary_bin<NT>(hist, k, sh, &bsel, &above, &cnt_b);
-    if (bsel != kNoBin) {
-      k_rem = k - above;
-      P.mode = 3;
-      P.vmin = st.vmin;
-      P.scale = scale;
-      if (cnt_b == k_rem) {  // the whole boundary bin is taken
-        P.bthr = static_cast<int>(bsel) - 1;
-        return P;
-      }
-      P.bthr = static_cast<int>(bsel);
-      if (cnt_b <= static_cast<uint32_t>(NT)) {
-        for (int i = threadIdx.x; i < n; i += NT) {
-          const uint32_t x = key[i];
-          if (is_cand(x) && x != kNanKey &&
-              value_bin(key_value(x), st.vmin, scale) == static_cast<int>(bsel)) {
-            const uint32_t j = atomicAdd(&sh.list_n, 1u);
-            if (j < static_cast<uint32_t>(NT)) {
-              list_key[j] = x;
-              list_idx[j] = static_cast<uint32_t>(i);
-            }
-          }
-        }
-        __syncthreads();
-        const uint32_t m = min(sh.list_n, static_cast<uint32_t>(NT));
-        // T threads rank one candidate (T m <= NT, T <= 32, aligned within a
-        // warp), each against every T-th other one, then sum over the T lanes.
-        uint32_t T = 32u;
-        while (T > 1u && T * m > static_cast<uint32_t>(NT)) T >>= 1;
-        const uint32_t cand = threadIdx.x / T, sub = threadIdx.x % T;
-        uint32_t rank = 0u, kt = 0u, it = 0u;
-        if (cand < m) {
-          kt = list_key[cand];
-          it = list_idx[cand];
-          for (uint32_t j = sub; j < m; j += T) {
-            const uint32_t kj = list_key[j];
-            rank += (kj > kt || (kj == kt && list_idx[j] < it)) ? 1u : 0u;
-          }
-        }
-        for (uint32_t off = T >> 1; off > 0u; off >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off);
-        if (cand < m && sub == 0u && rank < k_rem) key[it] = mark;
-        __syncthreads();
-        return P;
-      }
-      // Too many candidates in the bin: exact search inside its key range.
-      uint32_t blo = 0xFFFFFFFFu, bhi = 0u;
-      for (int i = threadIdx.x; i < n; i += NT) {
-        const uint32_t x = key[i];
-        if (is_cand(x) && x != kNanKey &&
-            value_bin(key_value(x), st.vmin, scale) == static_cast<int>(bsel)) {
-          blo = min(blo, x);
-          bhi = max(bhi, x);
-        }
-      }
-      block_minmax<NT>(blo, bhi, &lo, &hi, sh);
-      cnt = cnt_b;
-    }
+    block_minmax<NT>(blo, bhi, &lo, &hi, sh);
+    cnt = cnt_b;
   }
   P.mode = 2;
-  window_search<NT>(key, n, lo, hi, k_rem, cnt, hist, sh, &P.T, &P.take, &P.cnt_eq);
+  window_search<NT>(key, n, lo, hi, k_rem, cnt, scratch, sh, &P.T, &P.take, &P.cnt_eq);
   return P;
 }
 
@@ -780,7 +699,7 @@ struct Picker {
         if (x > P.T) return true;
         if (x == P.T) return all_ties || (rank++ < P.take);
         return false;
-      case 3: return x != kNanKey && value_bin(key_value(x), P.vmin, P.scale) > P.bthr;
+      case 3: return x != kNanKey && P.bins.of(key_value(x)) > P.bthr;
       default: return false;
     }
   }
@@ -800,44 +719,78 @@ __device__ Picker make_picker(const uint32_t* key, int c0, int c1, const Plan& P
 }
 
 // The whole selection of slab s by one block of NT threads. smem holds
-// select_smem_words<NT>(n_past) words. Scores are read with plain loads (they
-// may have been written earlier in the same kernel).
+// select_smem_words<NT>(n_past, a.van_smem) words. Scores are read through L2
+// only (they may have been written earlier in the same kernel).
 template <int NT>
 __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelShared& sh) {
+  constexpr int kB = 8;  // score loads in flight per thread
   const int n_past = static_cast<int>(a.n_tokens - a.rp);
+  const int npad = (n_past + 3) & ~3;
   uint32_t* key = smem;
-  uint32_t* hist = smem + ((n_past + 3) & ~3);
-  uint32_t* list_key = hist + kSelectBins;
+  uint32_t* hist_t = smem + npad;
+  uint32_t* hist_v = hist_t + kSelectBins;
+  uint32_t* list_key = hist_v + kSelectBins;
   uint32_t* list_idx = list_key + NT;
+  // VaN goes to shared memory in the same pass as TaR when there is room,
+  // so that the VaN stage does not wait for a second round of loads.
+  float* vbuf = a.van_smem ? reinterpret_cast<float*>(list_idx + NT) : nullptr;
   const float* tar = a.tar + s * a.n_tokens;
   const float* van = a.van + s * a.n_tokens;
   const int chunk = (n_past + NT - 1) / NT;
   const int c0 = min(n_past, static_cast<int>(threadIdx.x) * chunk);
   const int c1 = min(n_past, c0 + chunk);
 
-  // VaN goes to shared memory in the same pass as TaR when there is room,
-  // so that the VaN stage does not wait for a second round of loads.
-  float* vbuf = a.van_smem ? reinterpret_cast<float*>(list_idx + NT) : nullptr;
+  for (int b = threadIdx.x; b < 2 * kSelectBins; b += NT) hist_t[b] = 0u;  // both histograms
+  __syncthreads();
+
+  // TaR keys and their histogram, and the range of VaN; kB loads of each
+  // kind in flight.
+  uint32_t nan_t = 0u;
+  float vmin = INFINITY, vmax = -INFINITY;
+  const Bins bt = tar_bins();
+  for (int i0 = threadIdx.x; i0 < n_past; i0 += kB * NT) {
+    float tv[kB], vv[kB];
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      const int i = i0 + b * NT;
+      tv[b] = i < n_past ? __ldcg(tar + i) : 0.0f;
+      vv[b] = i < n_past ? __ldcg(van + i) : 0.0f;
+    }
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      const int i = i0 + b * NT;
+      if (i >= n_past) break;
+      const float v = (a.neg_tar ? -tv[b] : tv[b]) + 0.0f;  // NaN stays NaN, -0 becomes +0
+      key[i] = score_key(v);
+      if (vbuf) vbuf[i] = vv[b];
+      if (v == v) {
+        atomicAdd(&hist_t[bt.of(v)], 1u);
+      } else {
+        ++nan_t;
+      }
+      const float u = (a.neg_van ? -vv[b] : vv[b]) + 0.0f;
+      if (u == u) {
+        vmin = fminf(vmin, u);
+        vmax = fmaxf(vmax, u);
+      }
+    }
+  }
+  // Its barriers also publish the keys and the histogram.
+  block_reduce3<NT>(&nan_t, &vmin, &vmax, sh);
+  const Bins bv = range_bins(vmin, vmax);
 
   // TaR stage over all past tokens.
-  Stats st{INFINITY, -INFINITY, 0u};
-  for (int i = threadIdx.x; i < n_past; i += NT) {
-    const float v = (a.neg_tar ? -tar[i] : tar[i]) + 0.0f;  // NaN stays NaN, -0 becomes +0
-    if (vbuf) vbuf[i] = van[i];
-    key[i] = score_key(v);
-    stats_add(st, v);
-  }
-  st = block_stats<NT>(st, sh);
   Plan P = plan_stage<NT>(key, n_past, static_cast<uint32_t>(a.n_tar), static_cast<uint32_t>(n_past),
-                          st, kExcluded, hist, list_key, list_idx, sh);
+                          nan_t, bt, hist_t, hist_t, kExcluded, list_key, list_idx, sh);
   Picker pk = make_picker<NT>(key, c0, c1, P, kExcluded, sh);
-  Stats sv{INFINITY, -INFINITY, 0u};
-  for (int i0 = c0; i0 < c1; i0 += 8) {
-    float vb[8];  // issue the VaN loads of 8 tokens before using any
+  // Mark TaR picks; the other past tokens take their VaN key, binned.
+  uint32_t nan_v = 0u;
+  for (int i0 = c0; i0 < c1; i0 += kB) {
+    float vb[kB];  // issue the VaN loads of kB tokens before using any
 #pragma unroll
-    for (int b = 0; b < 8; ++b) vb[b] = (i0 + b < c1) ? (vbuf ? vbuf[i0 + b] : van[i0 + b]) : 0.0f;
+    for (int b = 0; b < kB; ++b) vb[b] = (i0 + b < c1) ? (vbuf ? vbuf[i0 + b] : __ldcg(van + i0 + b)) : 0.0f;
 #pragma unroll
-    for (int b = 0; b < 8; ++b) {
+    for (int b = 0; b < kB; ++b) {
       const int i = i0 + b;
       if (i >= c1) break;
       if (pk.pick(key[i])) {
@@ -845,16 +798,20 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
       } else {
         const float v = (a.neg_van ? -vb[b] : vb[b]) + 0.0f;
         key[i] = score_key(v);
-        stats_add(sv, v);
+        if (v == v) {
+          atomicAdd(&hist_v[bv.of(v)], 1u);
+        } else {
+          ++nan_v;
+        }
       }
     }
   }
-  sv = block_stats<NT>(sv, sh);  // its barriers also publish the keys
+  nan_v = block_sum<NT>(nan_v, sh);  // its barriers also publish the keys and the histogram
 
   // VaN stage over the past tokens TaR left.
   const uint32_t n_rest = static_cast<uint32_t>(n_past - a.n_tar);
-  P = plan_stage<NT>(key, n_past, static_cast<uint32_t>(a.n_van), n_rest, sv, kTaken, hist,
-                     list_key, list_idx, sh);
+  P = plan_stage<NT>(key, n_past, static_cast<uint32_t>(a.n_van), n_rest, nan_v, bv, hist_v, hist_t,
+                     kTaken, list_key, list_idx, sh);
   pk = make_picker<NT>(key, c0, c1, P, kTaken, sh);
   for (int i = c0; i < c1; ++i)
     if (pk.pick(key[i])) key[i] = kTaken;
@@ -896,22 +853,338 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
   // guards only keep a broken count from writing outside this slab's row.
   for (int64_t j = threadIdx.x; j < a.rp; j += NT)
     if (total + j < a.budget) kept[total + j] = static_cast<int32_t>(n_past + j);
+  __syncthreads();  // the block's shared memory may be reused for the next slab
+}
+
+// ---------------------------------------------------------- selection, keys in registers
+// The same selection with each thread holding its contiguous chunk of at
+// most E past tokens in registers (chunk = ceil(n_past / NT)): every pass is
+// register arithmetic, a token's bins are computed once, the boundary bin's
+// candidates of a stage are collected while the stage's other tokens are
+// classified, and the output positions come from one block scan of the
+// threads' pick counts (chunks are in index order). For n_past <= NT * E.
+
+// Shared memory of select_slab_reg: hist_t[2048], hist_v[2048], list_key[NT],
+// list_idx[NT], two winner bitmaps of ceil(n_past / 32) words.
+template <int NT>
+__host__ __device__ constexpr size_t select_reg_smem_words(int64_t n_past) {
+  return 2 * kSelectBins + 2 * NT + 2 * static_cast<size_t>((n_past + 31) / 32);
+}
+
+// Exclusive prefix sum of v over the block's threads in thread order, with
+// the total, the min of lo and the max of hi over the block, in one pair of
+// barriers.
+template <int NT>
+__device__ uint32_t block_scan_minmax(uint32_t v, uint32_t* total, float* lo, float* hi, SelShared& sh) {
+  constexpr int W = NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t incl = warp_incl_scan(v);
+  float l = *lo, h = *hi;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
+    h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
+  }
+  if (lane == 31) sh.warp_a[warp] = incl;
+  if (lane == 0) {
+    sh.warp_f[warp] = l;
+    sh.warp_g[warp] = h;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t w = lane < W ? sh.warp_a[lane] : 0u;
+    const uint32_t wi = warp_incl_scan(w);
+    sh.warp_b[lane] = wi - w;
+    l = lane < W ? sh.warp_f[lane] : INFINITY;
+    h = lane < W ? sh.warp_g[lane] : -INFINITY;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
+      h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
+    }
+    if (lane == 31) sh.bcast[7] = wi;
+    if (lane == 0) {
+      sh.fcast[0] = l;
+      sh.fcast[1] = h;
+    }
+  }
+  __syncthreads();
+  const uint32_t out = sh.warp_b[warp] + incl - v;
+  *total = sh.bcast[7];
+  *lo = sh.fcast[0];
+  *hi = sh.fcast[1];
+  __syncthreads();
+  return out;
+}
+
+// One stage over the register-resident tokens: picks the k best (key desc,
+// index asc; NaN keys lowest) among the tokens whose bit is set in elig (bit
+// e: token i0 + e). n_cand candidates in the block, n_nan of them NaN, and
+// nan_before NaN candidates in lower-numbered threads. hist holds the
+// candidates' numbers in bins (built by the caller); scratch is 2048 words
+// that may be overwritten, winmap a zeroed bitmap of ceil(n_past/32) words.
+// Returns the picks as a bit mask. Block-uniform arguments except key, elig,
+// nan_before.
+template <int NT, int E>
+__device__ uint32_t stage_reg(const uint32_t (&key)[E], uint32_t elig, int i0, uint32_t k, uint32_t n_cand,
+                              uint32_t n_nan, uint32_t nan_before, Bins bins, const uint32_t* hist,
+                              uint32_t* scratch, uint32_t* list_key, uint32_t* list_idx, uint32_t* winmap,
+                              SelShared& sh) {
+  if (k == 0u) return 0u;
+  if (k >= n_cand) return elig;
+  const uint32_t n_num = n_cand - n_nan;
+  uint32_t pick = 0u;
+  if (k > n_num) {  // every number, then the lowest-index NaNs
+    const uint32_t take = k - n_num;
+    uint32_t r = nan_before;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      if (!((elig >> e) & 1u)) continue;
+      if (key[e] != kNanKey) {
+        pick |= 1u << e;
+      } else {
+        if (r < take) pick |= 1u << e;
+        ++r;
+      }
+    }
+    return pick;
+  }
+  uint32_t bsel, above, cnt_b;
+  boundary_bin<NT>(hist, k, sh, &bsel, &above, &cnt_b);
+  uint32_t k_rem = k - above;
+  if (bsel != kNoBin && cnt_b == k_rem) {  // the whole boundary bin is taken
+#pragma unroll
+    for (int e = 0; e < E; ++e)
+      if (((elig >> e) & 1u) && key[e] != kNanKey && bins.of(key_value(key[e])) >= static_cast<int>(bsel))
+        pick |= 1u << e;
+    return pick;
+  }
+  if (bsel != kNoBin && cnt_b <= static_cast<uint32_t>(NT)) {
+    if (threadIdx.x == 0) sh.list_n = 0u;
+    __syncthreads();
+    uint32_t in_bin = 0u;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      if (!((elig >> e) & 1u) || key[e] == kNanKey) continue;
+      const int b = bins.of(key_value(key[e]));
+      if (b > static_cast<int>(bsel)) {
+        pick |= 1u << e;
+      } else if (b == static_cast<int>(bsel)) {
+        in_bin |= 1u << e;
+        const uint32_t j = atomicAdd(&sh.list_n, 1u);
+        if (j < static_cast<uint32_t>(NT)) {
+          list_key[j] = key[e];
+          list_idx[j] = static_cast<uint32_t>(i0 + e);
+        }
+      }
+    }
+    __syncthreads();
+    const uint32_t m = min(sh.list_n, static_cast<uint32_t>(NT));
+    // T threads rank one candidate (T m <= NT, T <= 32, aligned within a
+    // warp), each against every T-th other one, then sum over the T lanes.
+    uint32_t T = 32u;
+    while (T > 1u && T * m > static_cast<uint32_t>(NT)) T >>= 1;
+    const uint32_t cand = threadIdx.x / T, sub = threadIdx.x % T;
+    uint32_t rank = 0u, kt = 0u, it = 0u;
+    if (cand < m) {
+      kt = list_key[cand];
+      it = list_idx[cand];
+      for (uint32_t j = sub; j < m; j += T) {
+        const uint32_t kj = list_key[j];
+        rank += (kj > kt || (kj == kt && list_idx[j] < it)) ? 1u : 0u;
+      }
+    }
+    for (uint32_t off = T >> 1; off > 0u; off >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off);
+    if (cand < m && sub == 0u && rank < k_rem) atomicOr(&winmap[it >> 5], 1u << (it & 31));
+    __syncthreads();
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      if (!((in_bin >> e) & 1u)) continue;
+      const int i = i0 + e;
+      if ((winmap[i >> 5] >> (i & 31)) & 1u) pick |= 1u << e;
+    }
+    return pick;
+  }
+  // Boundary bin too crowded: exact search over integer key windows.
+  uint32_t lo = 2u, hi = kTaken - 1u, cnt = n_num;
+  if (bsel != kNoBin) {
+    uint32_t blo = 0xFFFFFFFFu, bhi = 0u;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      if (!((elig >> e) & 1u) || key[e] == kNanKey) continue;
+      if (bins.of(key_value(key[e])) == static_cast<int>(bsel)) {
+        blo = min(blo, key[e]);
+        bhi = max(bhi, key[e]);
+      }
+    }
+    block_minmax<NT>(blo, bhi, &lo, &hi, sh);
+    cnt = cnt_b;
+  } else {
+    k_rem = k;
+  }
+  for (int round = 0; round < 8; ++round) {
+    if (lo == hi) break;
+    const uint64_t W = static_cast<uint64_t>(hi - lo) + 1u;
+    for (int b = threadIdx.x; b < kSelectBins; b += NT) scratch[b] = 0u;
+    __syncthreads();
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const uint32_t x = key[e];
+      if (((elig >> e) & 1u) && x >= lo && x <= hi)
+        atomicAdd(&scratch[(static_cast<uint64_t>(x - lo) * kSelectBins) / W], 1u);
+    }
+    __syncthreads();
+    uint32_t b2, above2, cnt2;
+    boundary_bin<NT>(scratch, k_rem, sh, &b2, &above2, &cnt2);
+    if (b2 == kNoBin) break;  // fewer candidates than k_rem: cannot happen
+    k_rem -= above2;
+    const uint32_t lo_b = lo + static_cast<uint32_t>((b2 * W + kSelectBins - 1) / kSelectBins);
+    const uint32_t hi_b = lo + static_cast<uint32_t>(((b2 + 1) * W + kSelectBins - 1) / kSelectBins) - 1u;
+    if (cnt2 == k_rem) {  // the whole window bin is taken: winners are keys >= lo_b
+      lo = hi = lo_b - 1u;
+      cnt = 0u;
+      k_rem = 0u;
+      break;
+    }
+    lo = lo_b;
+    hi = hi_b;
+    cnt = cnt2;
+  }
+  // Winners: keys above lo, and the k_rem lowest-index keys equal to lo
+  // (cnt of them; all when k_rem == cnt).
+  uint32_t eq = 0u;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    if (!((elig >> e) & 1u)) continue;
+    if (key[e] > lo) pick |= 1u << e;
+    if (key[e] == lo) eq |= 1u << e;
+  }
+  uint32_t tot;
+  uint32_t r = block_excl_scan<NT>(__popc(eq), &tot, sh);
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    if (!((eq >> e) & 1u)) continue;
+    if (r < k_rem) pick |= 1u << e;
+    ++r;
+  }
+  return pick;
+}
+
+template <int NT, int E>
+__device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, SelShared& sh) {
+  const int n_past = static_cast<int>(a.n_tokens - a.rp);
+  const int words = (n_past + 31) / 32;
+  uint32_t* hist_t = smem;
+  uint32_t* hist_v = hist_t + kSelectBins;
+  uint32_t* list_key = hist_v + kSelectBins;
+  uint32_t* list_idx = list_key + NT;
+  uint32_t* win_t = list_idx + NT;
+  uint32_t* win_v = win_t + words;
+  const float* tar = a.tar + s * a.n_tokens;
+  const float* van = a.van + s * a.n_tokens;
+  const int chunk = (n_past + NT - 1) / NT;  // <= E
+  const int i0 = min(n_past, static_cast<int>(threadIdx.x) * chunk);
+  const int cnt = min(n_past - i0, chunk);
+  const uint32_t mine = cnt >= 32 ? 0xFFFFFFFFu : ((1u << cnt) - 1u);
+
+  for (int b = threadIdx.x; b < 2 * kSelectBins; b += NT) hist_t[b] = 0u;  // both histograms
+  for (int b = threadIdx.x; b < 2 * words; b += NT) win_t[b] = 0u;          // both bitmaps
+  __syncthreads();
+
+  // Keys, TaR histogram, range of VaN. A warp's chunks are contiguous, so the
+  // loads of one e across the warp share cache lines (plain loads through L1).
+  // All of a thread's loads are issued before any result is used.
+  uint32_t tk[E], vk[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    tk[e] = e < cnt ? __float_as_uint(tar[i0 + e]) : 0u;
+    vk[e] = e < cnt ? __float_as_uint(van[i0 + e]) : 0u;
+  }
+  uint32_t nan_t = 0u;
+  float vmin = INFINITY, vmax = -INFINITY;
+  const Bins bt = tar_bins();
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const float t = __uint_as_float(tk[e]), u = __uint_as_float(vk[e]);
+    const float tv = (a.neg_tar ? -t : t) + 0.0f;  // NaN stays NaN, -0 becomes +0
+    const float vv = (a.neg_van ? -u : u) + 0.0f;
+    tk[e] = e < cnt ? score_key(tv) : kNanKey;
+    vk[e] = e < cnt ? score_key(vv) : kNanKey;
+    if (e < cnt) {
+      if (tv == tv) {
+        atomicAdd(&hist_t[bt.of(tv)], 1u);
+      } else {
+        ++nan_t;
+      }
+      if (vv == vv) {
+        vmin = fminf(vmin, vv);
+        vmax = fmaxf(vmax, vv);
+      }
+    }
+  }
+  uint32_t nan_t_all;
+  const uint32_t nan_t_before = block_scan_minmax<NT>(nan_t, &nan_t_all, &vmin, &vmax, sh);
+  const Bins bv = range_bins(vmin, vmax);
+
+  // TaR stage over all past tokens.
+  const uint32_t pick_t = stage_reg<NT, E>(tk, mine, i0, static_cast<uint32_t>(a.n_tar),
+                                           static_cast<uint32_t>(n_past), nan_t_all, nan_t_before, bt, hist_t,
+                                           hist_t, list_key, list_idx, win_t, sh);
+  // VaN histogram of the tokens TaR left.
+  const uint32_t rest = mine & ~pick_t;
+  uint32_t nan_v = 0u;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    if (!((rest >> e) & 1u)) continue;
+    if (vk[e] != kNanKey) {
+      atomicAdd(&hist_v[bv.of(key_value(vk[e]))], 1u);
+    } else {
+      ++nan_v;
+    }
+  }
+  uint32_t nan_v_all;
+  float d0 = 0.0f, d1 = 0.0f;
+  const uint32_t nan_v_before = block_scan_minmax<NT>(nan_v, &nan_v_all, &d0, &d1, sh);
+
+  // VaN stage over the past tokens TaR left.
+  const uint32_t pick_v = stage_reg<NT, E>(vk, rest, i0, static_cast<uint32_t>(a.n_van),
+                                           static_cast<uint32_t>(n_past - a.n_tar), nan_v_all, nan_v_before, bv,
+                                           hist_v, hist_t, list_key, list_idx, win_v, sh);
+
+  // Ascending kept indices: this thread's picks at the block prefix of the
+  // counts, then the recent frames.
+  const uint32_t pick = pick_t | pick_v;
+  uint32_t total;
+  uint32_t pos = block_excl_scan<NT>(__popc(pick), &total, sh);
+  int32_t* kept = a.kept + s * a.budget;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    if (!((pick >> e) & 1u)) continue;
+    if (pos < a.budget) kept[pos] = i0 + e;
+    ++pos;
+  }
+  // total == n_tar + n_van by construction; the guards only keep a broken
+  // count from writing outside this slab's row.
+  for (int64_t j = threadIdx.x; j < a.rp; j += NT)
+    if (total + j < a.budget) kept[total + j] = static_cast<int32_t>(n_past + j);
+  __syncthreads();  // the block's shared memory may be reused for the next slab
 }
 
 // ------------------------------------------------------------------ compaction
 // Sec. 3.1 / Algorithm 2 last step: dst row j of a slab = src row kept[j].
 // Half-warp hw (of n_hw) copies rows g = g_begin + hw, g_begin + hw + n_hw,
 // ... of the flattened (slab, j) range [g_begin, g_end), kU rows in flight.
-// Kept indices and source patch ids are read with plain loads (the kept
-// indices may have been written earlier in the same kernel). IDS: copy the
+// Kept indices are read through L2 only (they may have been written earlier
+// in the same kernel), source patch ids with plain loads. IDS: copy the
 // patch and frame ids of each row here too (else gather_ids does it).
 // JN > 0 (the step kernels): g runs over (slab, j) with j < jn kept rows per
 // slab, the kept stride staying a.budget; FIXED: the source row is
 // a.n_tokens - a.rp + j and kept is not read (the recent frames, j < rp,
 // written to rows budget - rp + j).
-template <int CPL, int kU, bool IDS = true, bool FIXED = false>
+template <int CPL, int kU, bool IDS = true, bool FIXED = false, bool LAST_USE = false>
 __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begin, int64_t g_end,
                                              int64_t hw, int64_t n_hw, int64_t jn = 0) {
+  const uint64_t pol = LAST_USE ? l2_evict_first() : 0;
   const int64_t per = jn > 0 ? jn : a.budget;  // (slab, j) rows per slab in g
   const int lane = threadIdx.x & 15;
   const int n_chunks = a.row_bytes / 16;
@@ -936,7 +1209,7 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
           n = static_cast<int>(a.n_tokens - a.rp + j);
           j += a.budget - a.rp;
         } else {
-          n = a.kept[(a.heads_per_kept > 1 ? s / a.heads_per_kept : s) * a.budget + j];
+          n = __ldcg(a.kept + (a.heads_per_kept > 1 ? s / a.heads_per_kept : s) * a.budget + j);
         }
         if (n >= a.cap) n = -1;  // never produced by the selection; ignore
       }
@@ -947,8 +1220,13 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
       for (int c = 0; c < CPL; ++c) {
         const int ch = lane + 16 * c;
         const bool ld = n >= 0 && ch < n_chunks;
-        kr[u][c] = ld ? ld_stream(ks + src_off + ch * 16) : make_uint4(0, 0, 0, 0);
-        vr[u][c] = ld ? ld_stream(vs + src_off + ch * 16) : make_uint4(0, 0, 0, 0);
+        if (LAST_USE) {  // the source rows are not read again in this pass
+          kr[u][c] = ld ? ld_stream(ks + src_off + ch * 16, pol) : make_uint4(0, 0, 0, 0);
+          vr[u][c] = ld ? ld_stream(vs + src_off + ch * 16, pol) : make_uint4(0, 0, 0, 0);
+        } else {
+          kr[u][c] = ld ? ld_stream(ks + src_off + ch * 16) : make_uint4(0, 0, 0, 0);
+          vr[u][c] = ld ? ld_stream(vs + src_off + ch * 16) : make_uint4(0, 0, 0, 0);
+        }
       }
     }
 #pragma unroll

@@ -171,25 +171,6 @@ size_t score_smem_bytes(int p, int D) {
   return b <= kScoreSmemLimit ? b : 0;  // 0: m is read through L1/L2 instead
 }
 
-int bulk_shape(int D, int is_bf16) {
-  const int n_chunks = D * (is_bf16 ? 2 : 4) / 16;
-  return n_chunks <= 8 ? 81 : n_chunks <= 16 ? 82 : n_chunks <= 32 ? 84 : n_chunks <= 64 ? 164 : 324;
-}
-
-size_t bulk_smem_bytes(int p, int D, int elem, int nst, int threads) {
-  const int shape = bulk_shape(D, elem == 2);
-  const int lpr = shape == 324 ? 32 : shape / 10;
-  const size_t rows = static_cast<size_t>(threads / 32) * (32 / lpr);  // one step of every warp
-  const size_t m = static_cast<size_t>((p * D + 31) & ~31) * sizeof(float);
-  return m + static_cast<size_t>(nst) * 2 * rows * D * elem;
-}
-
-int bulk_stages(int p, int D, int elem, int threads) {
-  for (int nst = kMaxStages; nst >= 2; --nst)
-    if (bulk_smem_bytes(p, D, elem, nst, threads) <= kBulkSmemMax) return nst;
-  return 0;
-}
-
 cudaError_t score_prepare(int, int) {
   cudaError_t e = prepare_t<uint16_t>();
   if (e == cudaSuccess) e = prepare_t<float>();

@@ -1,6 +1,7 @@
 // Step (iii) of the compression pass: the split-budget selection, one
 // 1024-thread block per (layer, KV head) slab. The algorithm (Sec. 3.3;
-// Algorithm 1 steps 3-5) is dev::select_slab in pass_device.cuh.
+// Algorithm 1 steps 3-5) is dev::select_slab_reg in pass_device.cuh (keys in
+// registers), or dev::select_slab (keys in shared memory) for larger slabs.
 #include "pass_device.cuh"
 
 namespace ipv {
@@ -12,6 +13,16 @@ __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a)
   pdl_trigger();
   pdl_wait();  // the scores come from the scoring kernel
   dev::select_slab<kSelectThreads>(a, blockIdx.x, sm_sel, sh);
+}
+
+// The same selection with every thread's share of the keys in registers,
+// for slabs of at most kSelectThreads * kSelectRegE past tokens.
+__global__ void __launch_bounds__(kSelectThreads, 1) select_reg_kernel(SelectArgs a) {
+  extern __shared__ uint32_t sm_sel[];
+  __shared__ dev::SelShared sh;
+  pdl_trigger();
+  pdl_wait();  // the scores come from the scoring kernel
+  dev::select_slab_reg<kSelectThreads, kSelectRegE>(a, blockIdx.x, sm_sel, sh);
 }
 
 __global__ void passthrough_kernel(int32_t* kept, int64_t n_slabs, int64_t n_tokens,
@@ -65,13 +76,21 @@ bool van_fits(int64_t n_past) {
 }  // namespace
 
 cudaError_t select_prepare(int64_t max_tokens) {
-  return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(select_smem_bytes(max_tokens)));
+  cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(select_smem_bytes(max_tokens)));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(
+      select_reg_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      static_cast<int>(dev::select_reg_smem_words<kSelectThreads>(kSelectThreads * kSelectRegE) * sizeof(uint32_t)));
 }
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st) {
   SelectArgs b = a;
   const int64_t n_past = a.n_tokens - a.rp;
+  if (n_past <= static_cast<int64_t>(kSelectThreads) * kSelectRegE) {
+    const size_t smem = dev::select_reg_smem_words<kSelectThreads>(n_past) * sizeof(uint32_t);
+    return launch(select_reg_kernel, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st, true, b);
+  }
   b.van_smem = van_fits(n_past) ? 1 : 0;
   const size_t smem = dev::select_smem_words<kSelectThreads>(n_past, b.van_smem != 0) * sizeof(uint32_t);
   return launch(select_kernel, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st, true, b);

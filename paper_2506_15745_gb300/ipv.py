@@ -17,7 +17,7 @@ IPV_OK, IPV_EINVAL, IPV_ENOINIT, IPV_ENOMEM, IPV_ECUDA, IPV_ETIMEOUT = range(6)
 IPV_BF16, IPV_F32 = 0, 1
 ABLATIONS = {"none": 0, "tar_reverse": 1, "van_reverse": 2, "tar_frame": 3, "uniform": 4}
 NUM_KERNELS = 7
-KERNEL_NAMES = ("recent_mean", "score", "select", "gather", "pipeline", "pool", "combine")
+KERNEL_NAMES = ("recent_mean", "score", "select", "gather", "fused", "pool", "combine")
 MAX_TOKENS = 49152
 MAX_POOL_FRAME_TOKENS = 4096
 
@@ -204,12 +204,12 @@ def append_frames(k: KV, v: KV, k_new, v_new, n_layers: int, n_kv_heads: int, he
 
 
 def set_wait_limit(polls: int) -> None:
-    """ipv_set_wait_limit: polls before a single-kernel-pass wait gives up (0: default)."""
+    """ipv_set_wait_limit: polls before a wait of the fused pass gives up (0: default)."""
     _check(load().ipv_set_wait_limit(int(polls)))
 
 
 def device_error() -> int:
-    """Timeout bits of the single-kernel pass since the last read (waits for the device)."""
+    """Timeout bits of the fused pass since the last read (waits for the device)."""
     out = ctypes.c_uint32(0)
     _check(load().ipv_device_error(ctypes.byref(out)))
     return out.value

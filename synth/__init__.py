@@ -213,16 +213,17 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
 
 
 def host_generate(w: Workload, stream: int = 0, n_frames: int | None = None,
-                  cap: int | None = None, slabs: int | None = None):
-    """K, V as numpy [S, cap, D] (float32, or uint16 bf16 bits), frames
-    0..n_frames-1 in rows 0..n_frames*p-1 (rest zero). For small cases."""
+                  cap: int | None = None, slabs: int | None = None, slab0: int = 0):
+    """K, V as numpy [S, cap, D] (float32, or uint16 bf16 bits) of slabs
+    slab0 .. slab0 + S - 1, frames 0..n_frames-1 in rows 0..n_frames*p-1
+    (rest zero). For small cases, or for slab ranges of a large one."""
     f = w.n_frames if n_frames is None else n_frames
-    S = w.slabs_per_stream if slabs is None else slabs
+    S = (w.slabs_per_stream - slab0) if slabs is None else slabs
     p, D = w.p, w.head_dim
     cap = f * p if cap is None else cap
     key = _key(w, stream)
     rho = patch_rho(w, stream).astype(np.float64)
-    s_idx = np.arange(S, dtype=np.uint64)[:, None, None]
+    s_idx = np.arange(slab0, slab0 + S, dtype=np.uint64)[:, None, None]
     q_idx = np.arange(p, dtype=np.uint64)[None, :, None]
     c_idx = np.arange(D // 4, dtype=np.uint64)[None, None, :]
     K = np.zeros((S, cap, D), np.float32)
@@ -231,7 +232,7 @@ def host_generate(w: Workload, stream: int = 0, n_frames: int | None = None,
     vp = value_params(w)
     vparams = None
     if vp is not None:  # per-slab sigma and beta of the slab's layer
-        layer = (np.arange(S) // w.n_kv_heads) % w.n_layers
+        layer = (np.arange(slab0, slab0 + S) // w.n_kv_heads) % w.n_layers
         vparams = (vp[0][layer].astype(np.float64), vp[1][layer].astype(np.float64))
     for t in range(f):
         tok = np.uint64(t * p) + q_idx

@@ -31,8 +31,11 @@ def test_reference_arm_line():
     assert d["n_gpus"] == 1 and d["steps"] == 2 and d["warmup"] == 1
     assert d["value"] > 0 and d["ms_per_step"] == d["value"]
     assert d["data"] == "synthetic" and d["config"]["workload"].startswith("tiny:")
+    w = synth.CONFIGS["tiny"]
+    assert d["config"] == bench.run_config(w, w.n_slabs, 1, 1, 1)  # the GPU arm's config object
     cpu = d["cpu_baseline"]
-    assert cpu["kind"] == "oracle" and cpu["cores"] >= 1 and cpu["value"] == d["value"] and cpu["sample"]
+    assert cpu["kind"] == "oracle" and cpu["cores"] >= 1 and cpu["value"] == d["value"]
+    assert cpu["sample"].startswith("every one of the 2 slabs")  # measured whole passes
     assert d["e2e"] == {"value": d["value"], "unit": "ms", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
 
@@ -65,3 +68,9 @@ def test_ablation_needs_a_per_head_raw_van_workload():
     for cfg in ("llava_pool", "llava_shared"):
         out = _run(["--config", cfg, "--ablation", "uniform"])
         assert out.returncode == 2 and "--ablation" in out.stderr
+
+
+def test_workload_strings_fit_the_record():
+    """The driver's record keeps 120 characters of config.workload."""
+    for w in synth.CONFIGS.values():
+        assert len(bench.workload_desc(w)) <= 120, w.name

@@ -57,6 +57,8 @@ def check_pass(cache, L, H, N, gh, gw, budget, alpha, pid_valid, slabs=None):
     v_src = to_np(cache.v_live.index_select(0, sel_t))
     pid_src = (to_np(cache.pid_live.index_select(0, sel_t))
                if (pid_valid and cache.pid is not None) else None)
+    fid_src = (cache.fid[cache.cur].index_select(0, sel_t).cpu().numpy()
+               if (pid_valid and cache.fid is not None) else None)
     k_struct, v_struct = cache.structs(pid_valid)
     tar_g = torch.empty((S, N), dtype=torch.float32, device="cuda")
     van_g = torch.empty_like(tar_g)
@@ -90,6 +92,11 @@ def check_pass(cache, L, H, N, gh, gw, budget, alpha, pid_valid, slabs=None):
         want = (np.take_along_axis(pid_src, kept_np, 1) if pid_src is not None
                 else (kept_np % p).astype(np.uint16))
         assert np.array_equal(pd, want)
+    if cache.fid is not None:  # frame ids travel with their rows too
+        fd = cache.fid[cache.cur].index_select(0, sel_t).cpu().numpy()[:, :budget]
+        want = (np.take_along_axis(fid_src, kept_np, 1) if fid_src is not None
+                else (kept_np // p).astype(np.int32))
+        assert np.array_equal(fd, want)
     return errs, n_diff
 
 
@@ -209,6 +216,76 @@ def test_select_exact_on_ties_nan_and_signed_zero():
         assert np.array_equal(to_np(kept), want), (budget, alpha)
 
 
+def test_select_exact_when_boundary_bins_overflow():
+    """Step (iii) on crafted scores whose boundary bin holds thousands of
+    close, distinct values (and ties): the selection's exact search over key
+    windows, bit-exact against the oracle."""
+    rng = np.random.default_rng(8)
+    S, f, p = 3, 64, 256
+    N = f * p
+    r = oracle.recent_frames(f)
+    n_past = N - r * p
+    init_for(S, N, 64, p, "f32")
+    tar = rng.uniform(-1.0, 0.2, size=(S, N)).astype(np.float32)
+    van = rng.uniform(0.0, 0.9, size=(S, N)).astype(np.float32)
+    # slab 0: 4000 TaR values within 1e-4 (one bin of the [-1, 1] map), 500 above
+    idx = rng.permutation(n_past)
+    tar[0, idx[:4000]] = (0.3 + rng.integers(0, 3000, 4000) * 3e-8).astype(np.float32)
+    tar[0, idx[4000:4500]] = rng.uniform(0.5, 1.0, 500).astype(np.float32)
+    # slab 1: VaN of 6000 tokens within 1e-3 of 1, 1000 spread above, one at 1000
+    tar[1, :2000] = 0.9  # TaR takes these (ties broken by index)
+    van[1, :2000] = 0.1
+    idx = 2000 + rng.permutation(n_past - 2000)
+    van[1, idx[:6000]] = (1.0 + rng.integers(0, 8000, 6000) * 1.25e-7).astype(np.float32)
+    van[1, idx[6000:7000]] = rng.uniform(10.0, 100.0, 1000).astype(np.float32)
+    van[1, idx[7000]] = 1000.0
+    # slab 2: both, with NaN and signed zeros in the clusters
+    tar[2] = tar[0]
+    van[2] = van[1]
+    tar[2, idx[:200]] = np.nan
+    van[2, idx[200:400]] = -0.0
+    for budget, alpha in [(8096, 0.5), (12288, 0.3), (6000, 0.6)]:
+        kept = torch.empty((S, budget), dtype=torch.int32, device="cuda")
+        ipv.select(torch.from_numpy(tar).cuda(), torch.from_numpy(van).cuda(), S, N, 1, p,
+                   budget, alpha, kept)
+        want = oracle.select(tar.astype(np.float64), van.astype(np.float64), N, p, r, budget,
+                             float(np.float32(alpha)))
+        assert np.array_equal(to_np(kept), want), (budget, alpha)
+
+
+def test_fused_selection_fallback_matches_steps():
+    """V norms that crowd one bin of the VaN map: the fused pass's 512-thread
+    selection takes the exact window search (the step kernels' 1024-thread
+    block as well in one slab, direct ranking in the other); indices and
+    bytes must agree bit for bit."""
+    S, f, gh, gw, D = 2, 256, 4, 4, 64
+    w = synth.Workload("crowded", 1, S, D, "f32", gh, gw, f, 128 * gh * gw, 0.5, seed=3)
+    p, N = w.p, w.n_tokens
+    K, V = synth.host_generate(w)
+    rng = np.random.default_rng(9)
+    r = oracle.recent_frames(f)
+    n_past = N - r * p
+    for s, n_cluster in ((0, 2600), (1, 800)):
+        u = V[s, :n_past] / np.linalg.norm(V[s, :n_past], axis=1, keepdims=True)
+        norm = rng.uniform(0.2, 0.5, n_past)
+        idx = rng.permutation(n_past)
+        norm[idx[:n_cluster]] = 1.0 + rng.integers(0, 4000, n_cluster) * 1e-6
+        norm[idx[n_cluster:n_cluster + 300]] = rng.uniform(2.0, 100.0, 300)
+        norm[idx[n_cluster + 300]] = 1000.0
+        V[s, :n_past] = (u * norm[:, None]).astype(np.float32)
+
+    def make_cache():
+        c = PingPongCache(S, N, D, "f32", patch_ids=True)
+        c.k[0] = to_dev(K, "f32")
+        c.v[0] = to_dev(V, "f32")
+        return c
+
+    (kp, cp), (ks, cs) = _run_both(w, 1, make_cache, pid_valid=False, passes=1)
+    B = w.budget
+    assert torch.equal(kp, ks)
+    assert torch.equal(cp.v[1, :, :B], cs.v[1, :, :B])
+
+
 def test_invalid_arguments_are_rejected():
     S, f, gh, gw, D = 2, 8, 4, 4, 64
     p, N = gh * gw, f * gh * gw
@@ -274,45 +351,48 @@ def test_full_config(name):
 
 
 def test_streaming_run():
-    """1 h at 1 fps at the LLaVA shape: 16 frames appended per step, a pass
-    whenever the cache holds 9408 tokens. Every pass keeps the invariants; the
-    first, a middle and the last pass are checked against the oracle on 16
-    sampled slabs (past rows then carry patch ids from earlier passes)."""
+    """1 h at 1 fps at the LLaVA shape (Algorithm 1's loop): 16 frames
+    appended per step through ipv_append_frames (patch ids and frame ids
+    numbered on the device), a pass whenever the cache holds 9408 tokens.
+    Every pass keeps the invariants; 10 evenly spaced passes of the 223 are
+    checked against the oracle on every slab (past rows then carry patch and
+    frame ids from earlier passes, and the ids must follow their rows)."""
     w = synth.CONFIGS["stream"]
-    S, p = w.slabs_per_stream, w.p
-    init_for(S, w.n_tokens, w.head_dim, p, w.dtype)
-    cache = PingPongCache(S, w.n_tokens, w.head_dim, w.dtype, patch_ids=True)
+    S, p, D, N, nf = w.slabs_per_stream, w.p, w.head_dim, w.n_tokens, w.append_frames
+    init_for(S, N, D, p, w.dtype)
+    cache = PingPongCache(S, N, D, w.dtype, patch_ids=True, frame_ids=True)
     gen = synth.DeviceGenerator(w, S)
+    k_new = torch.empty((S, nf * p, D), dtype=cache.k.dtype, device="cuda")
+    v_new = torch.empty_like(k_new)
     kept = torch.empty((S, w.budget), dtype=torch.int32, device="cuda")
-    n_passes = (w.stream_frames - w.n_frames) // w.append_frames + 1
-    check_at = {0, n_passes // 2, n_passes - 1}
-    sample = np.random.default_rng(0).choice(S, 16, replace=False)
+    n_passes = (w.stream_frames - w.n_frames) // nf + 1
+    check_at = set(np.linspace(0, n_passes - 1, 10).round().astype(int).tolist())
     r = ipv.recent_frames(w.n_frames)
     passes = frames = 0
-    first = True
     while frames < w.stream_frames:
-        nf = min(w.append_frames, w.stream_frames - frames)
-        row0 = cache.n_tokens
-        gen.fill(cache.k_live, cache.v_live, row0, nf)
-        cache.pid_live[:, row0:row0 + nf * p] = (
-            torch.arange(nf * p, device="cuda").remainder(p).to(torch.int16))
+        assert w.stream_frames - frames >= nf  # 3600 frames are 225 blocks of 16
+        gen.fill(k_new, v_new, 0, nf)
+        k, v = cache.structs(pid_valid=True)
+        ipv.append_frames(k, v, k_new, v_new, w.n_layers, w.n_kv_heads, D, cache.n_tokens, nf,
+                          w.grid_h, w.grid_w)
         cache.n_tokens += nf * p
         frames += nf
-        if cache.n_tokens >= w.n_tokens:
-            assert cache.n_tokens == w.n_tokens
+        if cache.n_tokens >= N:
+            assert cache.n_tokens == N
             if passes in check_at:
-                check_pass(cache, w.n_layers, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w,
-                           w.budget, w.tar_ratio, pid_valid=True, slabs=sample)
+                check_pass(cache, w.n_layers, w.n_kv_heads, N, w.grid_h, w.grid_w,
+                           w.budget, w.tar_ratio, pid_valid=True)
+                newest = cache.fid[cache.cur, :, w.budget - 1]
+                assert torch.all(newest == frames - 1)  # device numbering followed the stream
             else:
                 cache.compress(w.n_layers, w.n_kv_heads, w.grid_h, w.grid_w, w.budget,
                                w.tar_ratio, kept, pid_valid=True)
                 kn = kept
                 assert torch.all(kn[:, 1:] > kn[:, :-1])
-                assert torch.equal(kn[:, -r * p:], torch.arange(w.n_tokens - r * p, w.n_tokens,
-                                                                device="cuda", dtype=torch.int32).expand(S, -1))
+                assert torch.equal(kn[:, -r * p:], torch.arange(N - r * p, N, device="cuda",
+                                                                dtype=torch.int32).expand(S, -1))
             passes += 1
-            first = False
-    assert passes == n_passes == 223 and not first
+    assert passes == n_passes == 223 and len(check_at) == 10
 
 
 def test_large_config_sampled():
@@ -367,17 +447,19 @@ def test_max_tokens(dtype, budget, alpha):
 
 
 def _run_both(w, L, make_cache, pid_valid, passes=1):
-    """Run `passes` passes with the single-kernel pipeline and with the staged
-    kernels on identical inputs; return both (kept, cache) results."""
+    """Run `passes` passes with the fused kernel and with the step kernels on
+    identical inputs; return both (kept, cache) results."""
     out = []
     for single in (True, False):
         init_for(w_slabs(w, L), w.n_tokens, w.head_dim, w.p, w.dtype, single_kernel=single)
         cache = make_cache()
         kept = torch.empty((cache.n_slabs, w.budget), dtype=torch.int32, device="cuda")
         for _ in range(passes):
-            cache.n_tokens = w.n_tokens
-            cache.compress(L, w.n_kv_heads, w.grid_h, w.grid_w, w.budget, w.tar_ratio, kept,
-                           pid_valid=pid_valid)
+            cache.cur = 0  # the same source half every time
+            k, v = cache.structs(pid_valid=pid_valid)
+            ipv.compress(k, v, L, w.n_kv_heads, w.head_dim, w.n_tokens, w.grid_h, w.grid_w,
+                         w.budget, w.tar_ratio, kept)
+        cache.cur = k.cur
         torch.cuda.synchronize()
         assert ipv.device_error() == 0
         out.append((kept.clone(), cache))
@@ -389,13 +471,7 @@ def w_slabs(w, L):
     return L * w.n_kv_heads
 
 
-@pytest.mark.parametrize("name", ["llava", "qwen", "tiny"])
-def test_pipeline_matches_staged(name):
-    """The single-kernel pass and the four step kernels run the same device
-    arithmetic: indices, compacted rows and patch ids are bit-identical."""
-    w = synth.CONFIGS[name]
-    L = w.n_layers
-
+def _fresh_cache(w):
     def make_cache():
         c = PingPongCache(w.slabs_per_stream, w.n_tokens, w.head_dim, w.dtype, patch_ids=True)
         if w.dtype == "f32":
@@ -404,20 +480,56 @@ def test_pipeline_matches_staged(name):
             c.v[0] = to_dev(V, w.dtype)
         else:
             synth.device_generate(w, c.k[0], c.v[0])
+        c.k[1].fill_(-7.0)
+        c.v[1].fill_(-7.0)
+        c.pid[1].fill_(-1)
         return c
+    return make_cache
 
-    (kp, cp), (ks, cs) = _run_both(w, L, make_cache, pid_valid=False)
+
+FUSED_SHAPES = {
+    # name: (layers, KV heads, head_dim, dtype, grid, frames, budget frames, alpha)
+    "ragged_items": (3, 5, 128, "bf16", (13, 11), 24, 17, 0.45),  # p = 143: items of 15 and 16 patches
+    "one_patch": (2, 3, 64, "bf16", (1, 1), 40, 30, 0.5),          # p = 1: one score item per slab
+    "wide_rows_f32": (2, 2, 512, "f32", (6, 7), 16, 11, 0.6),      # 2 KB rows: fewer patches per item
+    "many_slabs": (40, 8, 64, "bf16", (4, 4), 32, 20, 0.3),       # 320 slabs: owners take several
+    "alpha_extremes0": (2, 4, 96, "bf16", (5, 5), 20, 12, 0.0),
+    "alpha_extremes1": (2, 4, 96, "bf16", (5, 5), 20, 12, 1.0),
+}
+
+
+@pytest.mark.parametrize("name", ["llava", "qwen", "tiny"] + sorted(FUSED_SHAPES))
+def test_fused_matches_steps(name):
+    """The fused kernel and the four step kernels run the same device
+    arithmetic: indices, compacted rows and patch ids are bit-identical; the
+    fused result also passes the oracle checks."""
+    if name in FUSED_SHAPES:
+        L, H, D, dt, (gh, gw), f, bf, alpha = FUSED_SHAPES[name]
+        w = synth.Workload(name, L, H, D, dt, gh, gw, f, bf * gh * gw, alpha, seed=len(name))
+    else:
+        w = synth.CONFIGS[name]
+    L = w.n_layers
+    (kp, cp), (ks, cs) = _run_both(w, L, _fresh_cache(w), pid_valid=False, passes=2)
     B = w.budget
     assert torch.equal(kp, ks)
     assert cp.cur == cs.cur == 1
     assert torch.equal(cp.k[1, :, :B], cs.k[1, :, :B])
     assert torch.equal(cp.v[1, :, :B], cs.v[1, :, :B])
     assert torch.equal(cp.pid[1, :, :B], cs.pid[1, :, :B])
+    if w.n_slabs * w.n_tokens <= 400_000:  # small enough for the oracle
+        init_for(w_slabs(w, L), w.n_tokens, w.head_dim, w.p, w.dtype, single_kernel=True)
+        try:
+            cache = _fresh_cache(w)()
+            check_pass(cache, L, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w, B, w.tar_ratio,
+                       pid_valid=False)
+        finally:
+            torch.cuda.synchronize()
+            ipv.shutdown()
 
 
-def test_pipeline_repeated_passes_and_patch_ids():
-    """Back-to-back single-kernel passes reuse the queue state the previous
-    pass reset; with shuffled patch ids the result still equals the staged path."""
+def test_fused_falls_back_for_a_compacted_cache():
+    """A live half with patch ids (a cache compacted before) goes through the
+    step kernels under single_kernel = 1: the result equals the step path's."""
     S, f, gh, gw, D = 24, 16, 7, 7, 128
     w = synth.Workload("case", 1, S, D, "bf16", gh, gw, f, 500, 0.5, seed=21)
     p, N = w.p, w.n_tokens
@@ -436,18 +548,8 @@ def test_pipeline_repeated_passes_and_patch_ids():
         c.pid[0] = torch.from_numpy(pid.view(np.int16)).cuda()
         return c
 
-    results = []
-    for single in (True, False):
-        init_for(S, N, D, p, "bf16", single_kernel=single)
-        kept = torch.empty((S, w.budget), dtype=torch.int32, device="cuda")
-        c = make_cache()
-        for _ in range(5):  # identical input each time: cur reset to the source half
-            k_s, v_s = c.structs(pid_valid=True)
-            k_s.cur = v_s.cur = 0
-            ipv.compress(k_s, v_s, 1, S, D, N, gh, gw, w.budget, w.tar_ratio, kept)
-        torch.cuda.synchronize()
-        assert ipv.device_error() == 0
-        results.append((kept.clone(), c.k[1, :, :w.budget].clone(), c.pid[1, :, :w.budget].clone()))
-        ipv.shutdown()
-    for a, b in zip(*results):
-        assert torch.equal(a, b)
+    (kp, cp), (ks, cs) = _run_both(w, 1, make_cache, pid_valid=True, passes=3)
+    B = w.budget
+    assert torch.equal(kp, ks)
+    assert torch.equal(cp.k[1, :, :B], cs.k[1, :, :B])
+    assert torch.equal(cp.pid[1, :, :B], cs.pid[1, :, :B])

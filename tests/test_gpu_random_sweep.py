@@ -3,7 +3,7 @@
 Each case draws a shape (layers, KV heads, head_dim, element type, frame
 grid, frame count), a budget of whole frames, a TaR ratio and one of the
 pass's modes: per-head index sets on the step kernels (sometimes with the
-recent-frame count overridden) or on the single persistent kernel,
+recent-frame count overridden) or on the fused persistent kernel,
 layer-adaptive pooled VaN (Sec. 3.2, Algorithm 2), one index set per layer
 (Sec. 3.1, K[:, I, :]), both of the last two, or a variant of the ablation
 table (Sec. 4), Uniform Select included. The pass runs on a fresh cache;

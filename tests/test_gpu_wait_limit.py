@@ -1,9 +1,10 @@
-"""Failure detection of the single-kernel pass without a GPU fault: every
-wait in it is bounded. With a one-poll limit the waits for data that is not
-ready yet give up, set their bits in the device error word, and the pass
+"""Failure detection of the fused pass without a GPU fault: every wait in
+it is bounded. With a one-poll limit the waits for data that is not ready
+yet (a slab's scores before its selection, a selection before the slab's
+compaction) give up, set their bits in the device error word, and the pass
 ends; the host reads the bits, the context stays usable, and the next pass
-(default limit) starts from a clean queue state and gives the same result
-as before the failure."""
+(default limit) starts from clean counters and gives the same result as
+before the failure."""
 import numpy as np
 import pytest
 

@@ -71,3 +71,16 @@ def test_layer_varying_values():
     assert corr[0] > 0.5 and abs(corr[-1]) < 0.1 and corr[0] > corr[1] > corr[2]
     # defaults leave every layer at value_sigma with no field
     assert synth.value_params(synth.CONFIGS["llava"]) is None
+
+
+def test_host_generation_of_a_slab_range_is_a_slice_of_the_whole():
+    """Slabs generated from an offset (the reference arm generates ranges in
+    parallel) equal the same slabs of one whole generation."""
+    w = synth.Workload("rng", 3, 2, 64, "bf16", 3, 4, 5, 24, 0.5, seed=9)
+    K, V = synth.host_generate(w)
+    K2, V2 = synth.host_generate(w, slabs=3, slab0=2)
+    assert np.array_equal(K[2:5], K2) and np.array_equal(V[2:5], V2)
+    wp = synth.CONFIGS["llava_pool"].scaled(n_layers=3, n_frames=3, grid_h=3, grid_w=3, budget=18)
+    Kp, Vp = synth.host_generate(wp)
+    Kq, Vq = synth.host_generate(wp, slabs=5, slab0=6)  # per-layer value parameters follow the slab
+    assert np.array_equal(Kp[6:11], Kq) and np.array_equal(Vp[6:11], Vq)

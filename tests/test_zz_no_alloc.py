@@ -27,6 +27,25 @@ def _llava_case():
     return w, cache, False
 
 
+def _qwen_case():
+    """The Qwen2-VL-7B shape: about 29.4 MB of the 32 MiB array, the pass
+    closest to the limit that the header promises to accept."""
+    w = synth.CONFIGS["qwen"]
+    cache = PingPongCache(w.slabs_per_stream, w.n_tokens, w.head_dim, w.dtype, patch_ids=True)
+    synth.device_generate(w, cache.k[0], cache.v[0])
+    return w, cache, False
+
+
+def _f32_case():
+    """fp32 storage: 3 layers x 2 heads, D=64, 6x6 patches, 24 frames."""
+    w = synth.Workload("f32case", 3, 2, 64, "f32", 6, 6, 24, 600, 0.6, seed=7)
+    K, V = synth.host_generate(w)
+    cache = PingPongCache(w.slabs_per_stream, w.n_tokens, w.head_dim, w.dtype, patch_ids=True)
+    cache.k[0] = torch.from_numpy(K).cuda()
+    cache.v[0] = torch.from_numpy(V).cuda()
+    return w, cache, False
+
+
 def _shuffled_case():
     """2 layers x 3 heads, D=64 bf16, 7x7 patches, 16 frames, past rows
     shuffled together with their patch ids (a cache compacted before)."""
@@ -75,7 +94,7 @@ def _run_pair(w, cache, pid_valid):
 
 
 def test_static_matches_compress_two_calls():
-    for make in (_llava_case, _shuffled_case):
+    for make in (_llava_case, _qwen_case, _shuffled_case, _f32_case):
         w, cache, pid_valid = make()
         (kc, kdc, vdc, pc), (ks, kds, vds, ps) = _run_pair(w, cache, pid_valid)
         # Indices are integer work: bit-exact. Rows are copied bytes: bit-exact.
@@ -102,3 +121,35 @@ def test_static_rejects_a_pass_larger_than_its_array():
     assert ei.value.status == ipv.IPV_EINVAL
     assert "working memory" in str(ei.value)
     assert k.cur == 0 and v.cur == 0
+
+
+def test_static_rejects_slab_counts_whose_byte_count_would_wrap():
+    # 2^30 x 2^30 slabs of 4 tokens: the byte counts would wrap to 0 in 64
+    # bits; the pass must still be rejected before anything is enqueued.
+    fake = [0x100000 * (i + 1) for i in range(4)]
+    k = ipv.KV.from_tensors((fake[0], fake[1]), (None, None), 0)
+    v = ipv.KV.from_tensors((fake[2], fake[3]), (None, None), 0)
+    with pytest.raises(ipv.IpvError) as ei:
+        ipv.compress_static(k, v, "f32", 4, 0, 1 << 30, 1 << 30, 4, 4, 1, 1, 2, 0.5, 0x200000)
+    assert ei.value.status == ipv.IPV_EINVAL
+    assert k.cur == 0 and v.cur == 0
+
+
+def test_static_passes_a_cache_within_budget_through():
+    """n_tokens <= budget: kept = 0..n_tokens-1 padded with -1; the cache is
+    neither copied nor flipped."""
+    S, N, B, D = 6, 48, 60, 64
+    cache = PingPongCache(S, 64, D, "bf16", patch_ids=True)
+    cache.k[0].normal_()
+    cache.v[0].normal_()
+    cache.k[1].fill_(-3.0)
+    before = cache.k[1].clone()
+    kept = torch.full((S, B), -9, dtype=torch.int32, device="cuda")
+    k, v = cache.structs(pid_valid=False)
+    ipv.compress_static(k, v, "bf16", 64, 0, 3, 2, D, N, 4, 4, B, 0.5, kept)
+    torch.cuda.synchronize()
+    assert k.cur == 0 and v.cur == 0
+    want = torch.full((S, B), -1, dtype=torch.int32)
+    want[:, :N] = torch.arange(N, dtype=torch.int32)
+    assert torch.equal(kept.cpu(), want)
+    assert torch.equal(cache.k[1], before)
