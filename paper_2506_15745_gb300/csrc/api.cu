@@ -271,8 +271,9 @@ cudaError_t launch_shared_scores(const ipv::ScoreArgs& phys, int n_kv_heads, flo
 }
 
 // Work decomposition of the fused pass (window.cu). Tuning constants: score
-// items of at most kWinPatches patches, gather items of kWinRows selected
-// rows, and a lag of kWinLag slabs between a slab's score and gather items.
+// items of at most IPV_WIN_PATCHES patches, gather items of IPV_WIN_ROWS
+// selected rows, and a window of IPV_WIN_LAG slabs that scoring may run ahead
+// of compaction (the L2 holds about that many slabs' rows).
 #ifndef IPV_WIN_PATCHES
 #define IPV_WIN_PATCHES 16
 #endif
@@ -280,7 +281,7 @@ cudaError_t launch_shared_scores(const ipv::ScoreArgs& phys, int n_kv_heads, flo
 #define IPV_WIN_ROWS 512
 #endif
 #ifndef IPV_WIN_LAG
-#define IPV_WIN_LAG 4
+#define IPV_WIN_LAG 8
 #endif
 
 size_t fused_smem(const ipv::WinArgs& w) {

@@ -12,7 +12,10 @@ constexpr float kNormEps = 1e-12f;   // cos(a,b) = a.b / (max|a|,eps)(max|b|,eps
 #define IPV_SELECT_THREADS 1024
 #endif
 constexpr int kSelectThreads = IPV_SELECT_THREADS;  // threads of the step path's selection block
-constexpr int kSelectRegE = 16;  // past tokens per thread when the selection keeps its keys in registers
+#ifndef IPV_SELECT_REG_E
+#define IPV_SELECT_REG_E 16
+#endif
+constexpr int kSelectRegE = IPV_SELECT_REG_E;  // past tokens per thread when the selection keeps its keys in registers
 constexpr int kSelectBins = 2048;
 constexpr int64_t kMaxTokens = 49152;  // IPV_MAX_TOKENS: selection keys live in shared memory
 
@@ -274,15 +277,16 @@ cudaError_t launch_pool(const PoolArgs& a, cudaStream_t st, bool pdl);
 // Fused pass (window.cu): one cooperative persistent kernel, streaming
 // blocks and owner blocks. Its counters live in library scratch, are zero
 // before a launch and are reset by the kernel's last block.
-struct WinState {
-  unsigned head;      // next streaming ticket
+struct WinState {      // counters first: a failed launch clears them up to `error`
+  unsigned head;      // next score item (slab-major)
   unsigned sel_head;  // next slab for an owner block
   unsigned exited;    // blocks that have left
+  unsigned gat_low;   // slabs below have all their gather items handed out
   unsigned error;     // bit 0: an owner gave up waiting for its slab's scores,
-                      // bit 1: a gather item gave up waiting for its selection
-  unsigned pad[4];
+                      // bit 1: a streaming block gave up waiting for work
+  unsigned pad[3];
 };
-constexpr int kWinFlags = 2;  // per-slab words: score items done, selection done
+constexpr int kWinFlags = 3;  // per-slab words: score items done, selection done, gather items handed out
 constexpr size_t kWinSmemMax = 112 * 1024;  // two blocks per SM
 constexpr int kWinBlock = 512;  // threads of a fused-pass block
 constexpr int kWinRegE = 18;    // past tokens per owner thread: the selection's keys stay in registers
@@ -296,7 +300,8 @@ struct WinArgs {
   int n_si;          // score items per slab (patch ranges)
   int qmax;          // most patches in one score item
   int n_gi, rows_gi; // gather items per slab, selected rows per gather item
-  int lag;           // slabs between a slab's score items and its gather items
+  int lag;           // window: score items run at most this many slabs ahead of the
+                     // oldest slab whose gather items are not all handed out
   int n_stream, n_owner;  // blocks of each kind
   int64_t spin_limit;
 };

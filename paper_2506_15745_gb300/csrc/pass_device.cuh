@@ -498,7 +498,8 @@ __device__ void block_minmax(uint32_t lo, uint32_t hi, uint32_t* out_lo, uint32_
 // thread t owns the 2048/NT bins just below bin 2048 - t 2048/NT), the count
 // of candidates in higher bins and the bin's own count. kNoBin if the
 // histogram holds fewer than k.
-template <int NT>
+// COPIES > 1: the histogram is that many copies of 2048 bins, summed here.
+template <int NT, int COPIES = 1>
 __device__ void boundary_bin(const uint32_t* hist, uint32_t k, SelShared& sh, uint32_t* bsel,
                              uint32_t* above, uint32_t* cnt_b) {
   constexpr int BPT = kSelectBins / NT;
@@ -506,7 +507,9 @@ __device__ void boundary_bin(const uint32_t* hist, uint32_t k, SelShared& sh, ui
   uint32_t h[BPT], local = 0u;
 #pragma unroll
   for (int j = 0; j < BPT; ++j) {
-    h[j] = hist[top - j];
+    h[j] = 0u;
+#pragma unroll
+    for (int c = 0; c < COPIES; ++c) h[j] += hist[c * kSelectBins + top - j];
     local += h[j];
   }
   if (threadIdx.x == 0) sh.bcast[2] = kNoBin;  // published by the scan's barriers
@@ -864,11 +867,17 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
 // classified, and the output positions come from one block scan of the
 // threads' pick counts (chunks are in index order). For n_past <= NT * E.
 
-// Shared memory of select_slab_reg: hist_t[2048], hist_v[2048], list_key[NT],
-// list_idx[NT], two winner bitmaps of ceil(n_past / 32) words.
+// Histogram copies of the register selection: warp w adds into copy w mod
+// kHistCopies, so that tokens of a popular bin contend on fewer shared-memory
+// atomics (the copies are summed when the boundary bin is sought).
+constexpr int kHistCopies = 4;
+
+// Shared memory of select_slab_reg: hist_t[kHistCopies][2048],
+// hist_v[kHistCopies][2048], list_key[NT], list_idx[NT], two winner bitmaps
+// of ceil(n_past / 32) words.
 template <int NT>
 __host__ __device__ constexpr size_t select_reg_smem_words(int64_t n_past) {
-  return 2 * kSelectBins + 2 * NT + 2 * static_cast<size_t>((n_past + 31) / 32);
+  return 2 * kHistCopies * kSelectBins + 2 * NT + 2 * static_cast<size_t>((n_past + 31) / 32);
 }
 
 // Exclusive prefix sum of v over the block's threads in thread order, with
@@ -921,7 +930,7 @@ __device__ uint32_t block_scan_minmax(uint32_t v, uint32_t* total, float* lo, fl
 // index asc; NaN keys lowest) among the tokens whose bit is set in elig (bit
 // e: token i0 + e). n_cand candidates in the block, n_nan of them NaN, and
 // nan_before NaN candidates in lower-numbered threads. hist holds the
-// candidates' numbers in bins (built by the caller); scratch is 2048 words
+// candidates' numbers in bins (kHistCopies copies, built by the caller); scratch is 2048 words
 // that may be overwritten, winmap a zeroed bitmap of ceil(n_past/32) words.
 // Returns the picks as a bit mask. Block-uniform arguments except key, elig,
 // nan_before.
@@ -950,7 +959,7 @@ __device__ uint32_t stage_reg(const uint32_t (&key)[E], uint32_t elig, int i0, u
     return pick;
   }
   uint32_t bsel, above, cnt_b;
-  boundary_bin<NT>(hist, k, sh, &bsel, &above, &cnt_b);
+  boundary_bin<NT, kHistCopies>(hist, k, sh, &bsel, &above, &cnt_b);
   uint32_t k_rem = k - above;
   if (bsel != kNoBin && cnt_b == k_rem) {  // the whole boundary bin is taken
 #pragma unroll
@@ -1075,11 +1084,12 @@ __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, 
   const int n_past = static_cast<int>(a.n_tokens - a.rp);
   const int words = (n_past + 31) / 32;
   uint32_t* hist_t = smem;
-  uint32_t* hist_v = hist_t + kSelectBins;
-  uint32_t* list_key = hist_v + kSelectBins;
+  uint32_t* hist_v = hist_t + kHistCopies * kSelectBins;
+  uint32_t* list_key = hist_v + kHistCopies * kSelectBins;
   uint32_t* list_idx = list_key + NT;
   uint32_t* win_t = list_idx + NT;
   uint32_t* win_v = win_t + words;
+  const int copy = ((threadIdx.x >> 5) % kHistCopies) * kSelectBins;  // this warp's histogram copy
   const float* tar = a.tar + s * a.n_tokens;
   const float* van = a.van + s * a.n_tokens;
   const int chunk = (n_past + NT - 1) / NT;  // <= E
@@ -1087,8 +1097,8 @@ __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, 
   const int cnt = min(n_past - i0, chunk);
   const uint32_t mine = cnt >= 32 ? 0xFFFFFFFFu : ((1u << cnt) - 1u);
 
-  for (int b = threadIdx.x; b < 2 * kSelectBins; b += NT) hist_t[b] = 0u;  // both histograms
-  for (int b = threadIdx.x; b < 2 * words; b += NT) win_t[b] = 0u;          // both bitmaps
+  for (int b = threadIdx.x; b < 2 * kHistCopies * kSelectBins; b += NT) hist_t[b] = 0u;  // histograms
+  for (int b = threadIdx.x; b < 2 * words; b += NT) win_t[b] = 0u;                          // bitmaps
   __syncthreads();
 
   // Keys, TaR histogram, range of VaN. A warp's chunks are contiguous, so the
@@ -1112,7 +1122,7 @@ __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, 
     vk[e] = e < cnt ? score_key(vv) : kNanKey;
     if (e < cnt) {
       if (tv == tv) {
-        atomicAdd(&hist_t[bt.of(tv)], 1u);
+        atomicAdd(&hist_t[copy + bt.of(tv)], 1u);
       } else {
         ++nan_t;
       }
@@ -1137,7 +1147,7 @@ __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, 
   for (int e = 0; e < E; ++e) {
     if (!((rest >> e) & 1u)) continue;
     if (vk[e] != kNanKey) {
-      atomicAdd(&hist_v[bv.of(key_value(vk[e]))], 1u);
+      atomicAdd(&hist_v[copy + bv.of(key_value(vk[e]))], 1u);
     } else {
       ++nan_v;
     }

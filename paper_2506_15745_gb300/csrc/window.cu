@@ -11,16 +11,21 @@
 // Two kinds of blocks run together, one of each per SM (a cooperative launch
 // keeps them all resident, so that their waits on one another end):
 //
-//   streaming blocks take tickets from one counter in slab order. Ticket
-//     sequence t = 0, 1, ...: the score items of slab t (its past rows, one
-//     item per range of patches: rows f p + q of a cache that has never been
-//     compacted), then the gather items of slab t - lag (its selected past
-//     rows, copied to the other ping-pong half). lag slabs of score work
-//     cover the selection's latency. A score item computes m_q of its own
-//     patches from their r recent K rows (the step kernels' arithmetic), so
-//     no block waits for another's means; tickets are claimed two ahead, and
-//     the next score item's recent rows are copied into shared memory while
-//     the current item runs.
+//   streaming blocks work on two kinds of items. Score items (a slab's past
+//     rows, one item per range of patches: rows f p + q of a cache that has
+//     never been compacted) come from one counter in slab order; a score
+//     item computes m_q of its own patches from their r recent K rows (the
+//     step kernels' arithmetic), so no block waits for another's means.
+//     Gather items (a slab's selected past rows, copied to the other
+//     ping-pong half) come from a per-slab counter once the slab's
+//     selection is done. Warp 0 of a block picks the block's next item: a
+//     ready gather item first (the lowest such slab), else the score item it
+//     holds. A block claims its next score item ahead, and copies that
+//     item's recent rows into shared memory while the current item runs,
+//     only while it lies within `window` slabs of the oldest slab whose
+//     gather items are not all handed out: so the rows of at most about
+//     `window` slabs wait in L2 for their compaction. A block never waits
+//     while it holds a score item.
 //   owner blocks take slabs in order. For its slab an owner copies the
 //     recent rows (always kept) to their final place, waits until the slab's
 //     score items are done, and runs the split-budget selection (Sec. 3.3;
@@ -63,19 +68,19 @@ __device__ __forceinline__ void release_add(unsigned* p, unsigned v) {
   atomicAdd(p, v);
 }
 
-struct Item {  // a decoded ticket
-  int kind;    // 0 none (padding), 1 score, 2 gather
+__device__ __forceinline__ unsigned ld_relaxed(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+struct Item {  // a score item
+  int kind;    // 1
   int s, k;    // slab, item within the slab
 };
 
-__device__ __forceinline__ Item decode(const WinArgs& a, unsigned tk) {
-  const int per_t = a.n_si + a.n_gi;
-  const int t = static_cast<int>(tk / per_t), k = static_cast<int>(tk % per_t);
-  const int S = static_cast<int>(a.sc.n_slabs);
-  if (k < a.n_si) return t < S ? Item{1, t, k} : Item{0, 0, 0};
-  const int s = t - a.lag;
-  return (s >= 0 && s < S) ? Item{2, s, k - a.n_si} : Item{0, 0, 0};
-}
+// What a streaming block does next (decided by warp 0).
+enum { kIdle = 0, kGather = 1, kScoreHeld = 2, kScoreNew = 3, kExit = 4 };
 
 // Score item k of a slab covers patches [k p / n_si, (k + 1) p / n_si).
 __device__ __forceinline__ int item_q0(const WinArgs& a, int k) { return k * a.sc.p / a.n_si; }
@@ -176,19 +181,21 @@ template <typename T, int LPR, int CPL, int GCPL>
 __global__ void __launch_bounds__(kWinThreads, 2) window_kernel(WinArgs a) {
   extern __shared__ __align__(16) uint32_t sm[];
   __shared__ dev::SelShared sh;
-  __shared__ unsigned s_tk[3];
+  __shared__ unsigned s_tk[1];
+  __shared__ unsigned s_cmd[3];
   __shared__ int s_last;
   constexpr int kGU = GCPL >= 4 ? 1 : 4 / GCPL;  // rows in flight per half-warp
   WinState* st = a.state;
   const int S = static_cast<int>(a.sc.n_slabs);
   unsigned* s_count = a.flags;      // score items finished
   unsigned* x_done = a.flags + S;   // selection finished
+  unsigned* g_next = a.flags + 2 * S;  // gather items handed out
   const int64_t rp = static_cast<int64_t>(a.sc.r) * a.sc.p;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   if (blockIdx.x < a.n_stream) {
     // ------------------------------------------------------------ streaming
-    const int per_t = a.n_si + a.n_gi;
-    const unsigned total = static_cast<unsigned>(S + a.lag) * per_t;
+    const unsigned total_s = static_cast<unsigned>(S) * a.n_si;  // score tickets
     const int f_past = static_cast<int>((a.sc.n_tokens - rp) / a.sc.p);
     const int row_bytes = a.sc.D * static_cast<int>(sizeof(T));
     const int ms = a.sc.D + 4;  // padded m rows: lane groups of different patches hit different banks
@@ -197,56 +204,106 @@ __global__ void __launch_bounds__(kWinThreads, 2) window_kernel(WinArgs a) {
                      reinterpret_cast<char*>(sm) + static_cast<int64_t>(rec_rows) * row_bytes};
     float* mtab = reinterpret_cast<float*>(krec[1] + static_cast<int64_t>(rec_rows) * row_bytes);
     float* rinv = mtab + a.qmax * ms;
-    // Tickets are claimed two ahead: the recent rows of the next score item
-    // are fetched while the current item runs.
-    if (threadIdx.x == 0) {
-      s_tk[0] = atomicAdd(&st->head, 1u);
-      s_tk[1] = atomicAdd(&st->head, 1u);
-    }
-    __syncthreads();
-    unsigned cur = s_tk[0], nxt = s_tk[1];
-    int slot = 0, cur_buf = 0, fill = 0;
-    Item it = cur < total ? decode(a, cur) : Item{0, 0, 0};
-    if (it.kind == 1) {
-      prefetch_recent(a, it, krec[fill], row_bytes);
-      cur_buf = fill;
-      fill ^= 1;
-    }
-    while (cur < total) {  // block-uniform
-      if (threadIdx.x == 0) s_tk[(slot + 2) % 3] = atomicAdd(&st->head, 1u);
-      const Item nt = nxt < total ? decode(a, nxt) : Item{0, 0, 0};
-      int nxt_buf = 0;
-      if (nt.kind == 1) {
-        prefetch_recent(a, nt, krec[fill], row_bytes);
-        nxt_buf = fill;
-        fill ^= 1;
-      }
-      if (it.kind == 1) {
-        if (nt.kind == 1) {
-          asm volatile("cp.async.wait_group 1;" ::: "memory");  // this item's rows, not the next's
-        } else {
-          cp_async_wait_all();
+    const unsigned kNone = 0xFFFFFFFFu;
+    unsigned held = kNone;  // score ticket claimed ahead, its recent rows in krec[hbuf]
+    int hbuf = 0;
+    int64_t idle = 0;
+    for (;;) {
+      if (warp == 0) {
+        int kind = kIdle;
+        unsigned id = 0u, nxt = kNone;
+        // A ready gather item: lane l looks at slab gat_low + l.
+        const unsigned gl = ld_relaxed(&st->gat_low);
+        const unsigned sl = gl + lane;
+        const bool in = sl < static_cast<unsigned>(S);
+        const unsigned gn = in ? ld_relaxed(&g_next[sl]) : 0xFFFFFFFFu;
+        const bool ready = in && gn < static_cast<unsigned>(a.n_gi) && ld_acquire(&x_done[sl]) != 0u;
+        unsigned mask = __ballot_sync(0xffffffffu, ready);
+        while (mask) {
+          const int l = __ffs(mask) - 1;
+          unsigned c = 0u;
+          if (lane == l) c = atomicAdd(&g_next[sl], 1u);
+          c = __shfl_sync(0xffffffffu, c, l);
+          if (c < static_cast<unsigned>(a.n_gi)) {
+            kind = kGather;
+            id = (gl + l) * static_cast<unsigned>(a.n_gi) + c;
+            break;
+          }
+          mask &= mask - 1u;
         }
-        __syncthreads();
-        const int q0 = item_q0(a, it.k), nq = item_q0(a, it.k + 1) - q0;
-        item_mean<T, LPR, CPL>(a, nq, krec[cur_buf], rinv, mtab, ms);
-        dev::score_patch_rows<T, LPR, CPL>(a.sc, it.s, q0, nq, f_past, mtab, ms);
-      } else if (it.kind == 2) {
-        if (threadIdx.x == 0 && !wait_at_least(&x_done[it.s], 1u, a.spin_limit)) atomicOr(&st->error, 2u);
-        __syncthreads();
-        const int64_t j0 = static_cast<int64_t>(it.k) * a.rows_gi;
-        const int64_t j1 = min(a.se.budget - rp, j0 + a.rows_gi);
-        const int64_t base = static_cast<int64_t>(it.s) * a.se.budget;
-        dev::gather_range<GCPL, kGU, true, false, true>(a.ga, base + j0, base + j1, threadIdx.x >> 4,
-                                                        blockDim.x >> 4);
+        // Move the watermark over slabs whose gather items are all handed out.
+        const unsigned open = __ballot_sync(0xffffffffu, !(in && gn >= static_cast<unsigned>(a.n_gi)));
+        const unsigned skip = open ? static_cast<unsigned>(__ffs(open) - 1) : 32u;
+        if (lane == 0) {
+          if (skip > 0u) atomicMax(&st->gat_low, gl + skip);
+          // Else the held score item, or a new one within the window; and
+          // the next one ahead, within the window.
+          auto claim = [&]() -> unsigned {
+            const unsigned h = ld_relaxed(&st->head);
+            if (h >= total_s || h / a.n_si >= gl + skip + a.lag) return kNone;
+            const unsigned t = atomicAdd(&st->head, 1u);
+            return t < total_s ? t : kNone;
+          };
+          if (kind == kIdle) {
+            if (held != kNone) {
+              kind = kScoreHeld;
+              id = held;
+            } else if ((id = claim()) != kNone) {
+              kind = kScoreNew;
+            }
+            if (kind != kIdle) nxt = claim();
+          }
+          if (kind == kIdle && held == kNone && ld_relaxed(&st->head) >= total_s &&
+              gl + skip >= static_cast<unsigned>(S))
+            kind = kExit;
+          s_cmd[0] = static_cast<unsigned>(kind);
+          s_cmd[1] = id;
+          s_cmd[2] = nxt;
+        }
       }
       __syncthreads();
-      if (it.kind == 1 && threadIdx.x == 0) release_add(&s_count[it.s], 1u);
-      slot = (slot + 1) % 3;
-      cur = nxt;
-      it = nt;
-      cur_buf = nxt_buf;
-      nxt = s_tk[(slot + 1) % 3];
+      const int kind = static_cast<int>(s_cmd[0]);
+      const unsigned id = s_cmd[1], nxt = s_cmd[2];
+      if (kind == kExit) break;
+      if (kind == kIdle) {
+        if (++idle > a.spin_limit) {  // nothing became ready: give up rather than hang
+          if (threadIdx.x == 0) atomicOr(&st->error, 2u);
+          break;
+        }
+        __nanosleep(256);
+        __syncthreads();  // s_cmd is rewritten next round
+        continue;
+      }
+      idle = 0;
+      if (kind == kGather) {
+        const int s = static_cast<int>(id / a.n_gi), c = static_cast<int>(id % a.n_gi);
+        const int64_t j0 = static_cast<int64_t>(c) * a.rows_gi;
+        const int64_t j1 = min(a.se.budget - rp, j0 + a.rows_gi);
+        const int64_t base = static_cast<int64_t>(s) * a.se.budget;
+        dev::gather_range<GCPL, kGU, true, false, true>(a.ga, base + j0, base + j1, threadIdx.x >> 4,
+                                                        blockDim.x >> 4);
+        __syncthreads();
+        continue;
+      }
+      // A score item: its recent rows (copied now if they were not claimed
+      // ahead), and the next item's rows into the other buffer meanwhile.
+      const Item it{1, static_cast<int>(id / a.n_si), static_cast<int>(id % a.n_si)};
+      if (kind == kScoreNew) prefetch_recent(a, it, krec[hbuf], row_bytes);
+      if (nxt != kNone) {
+        const Item nt{1, static_cast<int>(nxt / a.n_si), static_cast<int>(nxt % a.n_si)};
+        prefetch_recent(a, nt, krec[hbuf ^ 1], row_bytes);
+        asm volatile("cp.async.wait_group 1;" ::: "memory");  // this item's rows, not the next's
+      } else {
+        cp_async_wait_all();
+      }
+      __syncthreads();
+      const int q0 = item_q0(a, it.k), nq = item_q0(a, it.k + 1) - q0;
+      item_mean<T, LPR, CPL>(a, nq, krec[hbuf], rinv, mtab, ms);
+      dev::score_patch_rows<T, LPR, CPL>(a.sc, it.s, q0, nq, f_past, mtab, ms);
+      __syncthreads();
+      if (threadIdx.x == 0) release_add(&s_count[it.s], 1u);
+      held = nxt;
+      if (nxt != kNone) hbuf ^= 1;
     }
     cp_async_wait_all();
   } else {
@@ -282,6 +339,7 @@ __global__ void __launch_bounds__(kWinThreads, 2) window_kernel(WinArgs a) {
     if (threadIdx.x == 0) {
       st->head = 0u;
       st->sel_head = 0u;
+      st->gat_low = 0u;
       st->exited = 0u;
     }
     __threadfence();
