@@ -348,6 +348,7 @@ struct SelShared {
   uint32_t bcast[8];
   float fcast[2];
   uint32_t list_n;
+  uint32_t list_cnt[2];  // the register selection's list counts, one per stage
 };
 
 // Shared memory of select_slab: keys[pad4(n_past)], hist_tar[2048],
@@ -364,19 +365,73 @@ __device__ __forceinline__ float key_value(uint32_t k) {  // inverse of score_ke
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
 }
 
+// 2^s as a float, for -126 <= s <= 127.
+__device__ __forceinline__ float exp2_int(int s) { return __uint_as_float(static_cast<uint32_t>(s + 127) << 23); }
+
 // A monotone non-decreasing map of a score (not NaN) to one of 2048 bins:
-// floor((v - lo) * scale), folded into [0, 2047] (scale 0: every value in bin 0).
+// floor(v mul) - off folded into [0, 2047], mul a power of two (or 0: every
+// value in bin 0) and off an integer. Because v mul is exact for the values
+// the bins resolve, the scores of bin b and above are those at or above
+// (b + off) / mul, so a stage's boundary bin turns into two integer key
+// thresholds (floor_key) and its tokens are classified by key compares.
 struct Bins {
-  float lo, scale;
+  float mul, off, inv;  // inv = 1 / mul (0 with mul)
   __device__ __forceinline__ int of(float v) const {
-    return static_cast<int>(fminf(fmaxf((v - lo) * scale, 0.0f), 2047.0f));
+    return static_cast<int>(fminf(fmaxf(floorf(v * mul) - off, 0.0f), 2047.0f));
+  }
+  __device__ __forceinline__ bool at_least(uint32_t key, int b) const { return of(key_value(key)) >= b; }
+  // The smallest number key (>= 2) whose score lies in bin b or above;
+  // kTaken if there is none. The estimate from the bin's lower edge is
+  // checked against its neighbour key; where rounding moved the edge, a
+  // binary search over the number keys (below the key of +inf, where bin is
+  // monotone) finds it. Block-uniform when b is.
+  __device__ uint32_t floor_key(int b) const {
+    constexpr uint32_t kInfKey = 0xFF800000u;  // score_key(+inf)
+    if (b <= 0) return 2u;
+    if (b >= kSelectBins || mul == 0.0f) return kTaken;
+    uint32_t x = score_key((static_cast<float>(b) + off) * inv);
+    x = min(max(x, 2u), kInfKey);
+    if (at_least(x, b) && (x == 2u || !at_least(x - 1u, b))) return x;
+    return search_key(*this, b);
+  }
+  __device__ static __noinline__ uint32_t search_key(Bins bins, int b) {
+    constexpr uint32_t kInfKey = 0xFF800000u;
+    if (!bins.at_least(kInfKey, b)) return kTaken;
+    uint32_t lo = 2u, hi = kInfKey;
+    while (lo < hi) {
+      const uint32_t mid = lo + (hi - lo) / 2u;
+      if (bins.at_least(mid, b)) {
+        hi = mid;
+      } else {
+        lo = mid + 1u;
+      }
+    }
+    return lo;
+  }
+  // The same edge as a score: bin(v) >= b exactly when v >= floor_value(b)
+  // (-inf for every number, NaN, which no score reaches, for none).
+  __device__ float floor_value(int b) const {
+    constexpr uint32_t kNegInfKey = 0x007FFFFFu;  // score_key(-inf)
+    const uint32_t x = floor_key(b);
+    if (x == kTaken) return __uint_as_float(0x7FC00000u);
+    return x <= kNegInfKey ? -INFINITY : key_value(x);
   }
 };
-__device__ __forceinline__ Bins tar_bins() { return Bins{-1.0f, 1024.0f}; }
+// TaR (a cosine, negated) in [-1, 1]: bins of width 1/1024.
+__device__ __forceinline__ Bins tar_bins() { return Bins{1024.0f, -1024.0f, 1.0f / 1024.0f}; }
+// VaN over its observed range [vmin, vmax]: the largest power-of-two scale
+// with (vmax - vmin) mul < 2048, kept below 2^21 |v| so that off stays an
+// exact integer. One bin when there is no finite range.
 __device__ __forceinline__ Bins range_bins(float vmin, float vmax) {
   const float range = vmax - vmin;
-  const float scale = static_cast<float>(kSelectBins) / range;
-  return Bins{vmin, (range > 0.0f && scale < INFINITY) ? scale : 0.0f};
+  if (!(range > 0.0f) || range == INFINITY) return Bins{0.0f, 0.0f, 0.0f};
+  const auto ilog2 = [](float x) {  // floor(log2 x) for normal x > 0; -127 below
+    return static_cast<int>((__float_as_uint(x) >> 23) & 0xFFu) - 127;
+  };
+  const int s = min(min(10 - ilog2(range), 20 - ilog2(fmaxf(fabsf(vmin), fabsf(vmax)))), 126);
+  const int sc = max(s, -126);
+  const float mul = exp2_int(sc);
+  return Bins{mul, floorf(vmin * mul), exp2_int(-sc)};
 }
 
 __device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v) {
@@ -389,7 +444,10 @@ __device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v) {
   return v;
 }
 
-// Exclusive prefix sum over the block's threads in thread order; *total gets the sum.
+// Exclusive prefix sum over the block's threads in thread order; *total gets
+// the sum. Every warp scans the warp totals itself, so the scan costs two
+// barriers (the second keeps warp_a from being rewritten by a next scan
+// before every warp has read it).
 template <int NT>
 __device__ uint32_t block_excl_scan(uint32_t v, uint32_t* total, SelShared& sh) {
   constexpr int W = NT / 32;
@@ -397,15 +455,10 @@ __device__ uint32_t block_excl_scan(uint32_t v, uint32_t* total, SelShared& sh) 
   const uint32_t incl = warp_incl_scan(v);
   if (lane == 31) sh.warp_a[warp] = incl;
   __syncthreads();
-  if (warp == 0) {
-    const uint32_t w = lane < W ? sh.warp_a[lane] : 0u;
-    const uint32_t wi = warp_incl_scan(w);
-    sh.warp_b[lane] = wi - w;
-    if (lane == 31) sh.bcast[7] = wi;
-  }
-  __syncthreads();
-  const uint32_t out = sh.warp_b[warp] + incl - v;
-  *total = sh.bcast[7];
+  const uint32_t wt = lane < W ? sh.warp_a[lane] : 0u;
+  const uint32_t wi = warp_incl_scan(wt);
+  *total = __shfl_sync(0xffffffffu, wi, 31);
+  const uint32_t out = __shfl_sync(0xffffffffu, wi - wt, warp) + incl - v;
   __syncthreads();
   return out;
 }
@@ -437,26 +490,47 @@ __device__ void block_reduce3(uint32_t* cnt, float* lo, float* hi, SelShared& sh
     sh.warp_g[warp] = h;
   }
   __syncthreads();
-  if (warp == 0) {
-    c = lane < W ? sh.warp_a[lane] : 0u;
-    l = lane < W ? sh.warp_f[lane] : INFINITY;
-    h = lane < W ? sh.warp_g[lane] : -INFINITY;
+  // Every warp reduces the warp partials itself.
+  c = lane < W ? sh.warp_a[lane] : 0u;
+  l = lane < W ? sh.warp_f[lane] : INFINITY;
+  h = lane < W ? sh.warp_g[lane] : -INFINITY;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      c += __shfl_xor_sync(0xffffffffu, c, off);
-      l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
-      h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
-    }
-    if (lane == 0) {
-      sh.bcast[5] = c;
-      sh.fcast[0] = l;
-      sh.fcast[1] = h;
-    }
+  for (int off = 16; off > 0; off >>= 1) {
+    c += __shfl_xor_sync(0xffffffffu, c, off);
+    l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
+    h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
+  }
+  *cnt = c;
+  *lo = l;
+  *hi = h;
+  __syncthreads();
+}
+
+// Block-wide min of *lo and max of *hi (every thread gets them); two barriers.
+template <int NT>
+__device__ void block_range(float* lo, float* hi, SelShared& sh) {
+  constexpr int W = NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float l = *lo, h = *hi;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
+    h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
+  }
+  if (lane == 0) {
+    sh.warp_f[warp] = l;
+    sh.warp_g[warp] = h;
   }
   __syncthreads();
-  *cnt = sh.bcast[5];
-  *lo = sh.fcast[0];
-  *hi = sh.fcast[1];
+  l = lane < W ? sh.warp_f[lane] : INFINITY;
+  h = lane < W ? sh.warp_g[lane] : -INFINITY;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
+    h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
+  }
+  *lo = l;
+  *hi = h;
   __syncthreads();
 }
 
@@ -499,10 +573,18 @@ __device__ void block_minmax(uint32_t lo, uint32_t hi, uint32_t* out_lo, uint32_
 // of candidates in higher bins and the bin's own count. kNoBin if the
 // histogram holds fewer than k.
 // COPIES > 1: the histogram is that many copies of 2048 bins, summed here.
+// Two barriers: bcast[2..4] and fcast are written only between them, and
+// every thread reads them before it can reach the first barrier of a next
+// call. With bins, the thread that finds the bin also turns its edges into
+// scores (*v_lo = bins.floor_value(bin), *v_hi = that of bin + 1); *total
+// gets the histogram's total.
 template <int NT, int COPIES = 1>
 __device__ void boundary_bin(const uint32_t* hist, uint32_t k, SelShared& sh, uint32_t* bsel,
-                             uint32_t* above, uint32_t* cnt_b) {
+                             uint32_t* above, uint32_t* cnt_b, const Bins* bins = nullptr,
+                             float* v_lo = nullptr, float* v_hi = nullptr, uint32_t* total = nullptr) {
   constexpr int BPT = kSelectBins / NT;
+  constexpr int W = NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int top = kSelectBins - 1 - BPT * static_cast<int>(threadIdx.x);
   uint32_t h[BPT], local = 0u;
 #pragma unroll
@@ -512,23 +594,49 @@ __device__ void boundary_bin(const uint32_t* hist, uint32_t k, SelShared& sh, ui
     for (int c = 0; c < COPIES; ++c) h[j] += hist[c * kSelectBins + top - j];
     local += h[j];
   }
-  if (threadIdx.x == 0) sh.bcast[2] = kNoBin;  // published by the scan's barriers
-  uint32_t tot;
-  uint32_t run = block_excl_scan<NT>(local, &tot, sh);
+  const uint32_t incl = warp_incl_scan(local);
+  if (lane == 31) sh.warp_a[warp] = incl;
+  __syncthreads();
+  const uint32_t wt = lane < W ? sh.warp_a[lane] : 0u;
+  const uint32_t wi = warp_incl_scan(wt);
+  const uint32_t tot = __shfl_sync(0xffffffffu, wi, 31);
+  uint32_t run = __shfl_sync(0xffffffffu, wi - wt, warp) + incl - local;
+  const bool finder = run < k && k <= run + local;  // the one thread holding the k-th
+  int b = 0;
+  if (finder) {
 #pragma unroll
-  for (int j = 0; j < BPT; ++j) {
-    if (run < k && k <= run + h[j]) {
-      sh.bcast[2] = static_cast<uint32_t>(top - j);
-      sh.bcast[3] = run;
-      sh.bcast[4] = h[j];
+    for (int j = 0; j < BPT; ++j) {
+      if (run < k && k <= run + h[j]) {
+        b = top - j;
+        sh.bcast[2] = static_cast<uint32_t>(b);
+        sh.bcast[3] = run;
+        sh.bcast[4] = h[j];
+      }
+      run += h[j];
     }
-    run += h[j];
+  }
+  if (bins) {  // lanes 0 and 1 of the finder's warp compute the two edges side by side
+    const unsigned fm = __ballot_sync(0xffffffffu, finder);
+    if (fm) {
+      const int bb = __shfl_sync(0xffffffffu, b, __ffs(fm) - 1);
+      if (lane < 2) sh.fcast[lane] = bins->floor_value(bb + lane);
+    }
   }
   __syncthreads();
-  *bsel = sh.bcast[2];
-  *above = sh.bcast[3];
-  *cnt_b = sh.bcast[4];
-  __syncthreads();
+  if (total) *total = tot;
+  if (k == 0u || tot < k) {
+    *bsel = kNoBin;
+    *above = 0u;
+    *cnt_b = 0u;
+  } else {
+    *bsel = sh.bcast[2];
+    *above = sh.bcast[3];
+    *cnt_b = sh.bcast[4];
+    if (bins) {
+      *v_lo = sh.fcast[0];
+      *v_hi = sh.fcast[1];
+    }
+  }
 }
 
 // Exact threshold search over integer key windows, from the window [lo, hi]
@@ -859,171 +967,172 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
   __syncthreads();  // the block's shared memory may be reused for the next slab
 }
 
-// ---------------------------------------------------------- selection, keys in registers
-// The same selection with each thread holding its contiguous chunk of at
-// most E past tokens in registers (chunk = ceil(n_past / NT)): every pass is
-// register arithmetic, a token's bins are computed once, the boundary bin's
-// candidates of a stage are collected while the stage's other tokens are
-// classified, and the output positions come from one block scan of the
-// threads' pick counts (chunks are in index order). For n_past <= NT * E.
+// ---------------------------------------------------------- selection, scores in registers
+// The same selection with the past tokens' scores in registers: thread t of
+// NT holds tokens t, t + NT, t + 2 NT, ... (at most E; bit j of a thread's
+// masks is token j NT + t, row j). Loads are coalesced; a stage's tokens
+// are classified against its boundary bin by two float compares (the bin's
+// edges as scores); the boundary bin's candidates are collected and ranked
+// exactly; every step that needs index order (the kept order, lowest-index
+// ties and NaNs) works on bitmaps whose word j W + w is warp w's ballot over
+// row j, so that word order is index order. For n_past <= NT * E.
 
 // Histogram copies of the register selection: warp w adds into copy w mod
 // kHistCopies, so that tokens of a popular bin contend on fewer shared-memory
 // atomics (the copies are summed when the boundary bin is sought).
 constexpr int kHistCopies = 4;
 
+// Above this many rows the VaN scores wait out the TaR stage in shared
+// memory, so that the stage has the registers it needs.
+constexpr int kRegStashRows = 10;
+
 // Shared memory of select_slab_reg: hist_t[kHistCopies][2048],
-// hist_v[kHistCopies][2048], list_key[NT], list_idx[NT], two winner bitmaps
-// of ceil(n_past / 32) words.
-template <int NT>
-__host__ __device__ constexpr size_t select_reg_smem_words(int64_t n_past) {
-  return 2 * kHistCopies * kSelectBins + 2 * NT + 2 * static_cast<size_t>((n_past + 31) / 32);
+// hist_v[kHistCopies][2048], list_key[NT], list_idx[NT], three bitmaps of
+// E NT / 32 words (the two stages' boundary-bin winners, and a scratch one
+// for index-order ranks and the picks) and, above kRegStashRows rows, the
+// VaN scores (E NT words).
+template <int NT, int E>
+__host__ __device__ constexpr size_t select_reg_smem_words() {
+  return 2 * kHistCopies * kSelectBins + 2 * NT + 3 * (E * NT / 32) + (E > kRegStashRows ? E * NT : 0);
 }
 
-// Exclusive prefix sum of v over the block's threads in thread order, with
-// the total, the min of lo and the max of hi over the block, in one pair of
-// barriers.
-template <int NT>
-__device__ uint32_t block_scan_minmax(uint32_t v, uint32_t* total, float* lo, float* hi, SelShared& sh) {
+// The `take` lowest-index tokens among those flagged in f (bit j: token
+// j NT + t; rows j < J), as a mask. bits is scratch of J NT / 32 words.
+// Block-uniform take and J.
+template <int NT, int E>
+__device__ __noinline__ uint32_t lowest_index(uint32_t f, uint32_t take, int J, uint32_t* bits, SelShared& sh) {
   constexpr int W = NT / 32;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const uint32_t incl = warp_incl_scan(v);
-  float l = *lo, h = *hi;
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
-    h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
-  }
-  if (lane == 31) sh.warp_a[warp] = incl;
-  if (lane == 0) {
-    sh.warp_f[warp] = l;
-    sh.warp_g[warp] = h;
+  for (int j = 0; j < E; ++j) {
+    const uint32_t b = __ballot_sync(0xffffffffu, (f >> j) & 1u);
+    if (j < J && lane == 0) bits[j * W + warp] = b;
   }
   __syncthreads();
-  if (warp == 0) {
-    const uint32_t w = lane < W ? sh.warp_a[lane] : 0u;
-    const uint32_t wi = warp_incl_scan(w);
-    sh.warp_b[lane] = wi - w;
-    l = lane < W ? sh.warp_f[lane] : INFINITY;
-    h = lane < W ? sh.warp_g[lane] : -INFINITY;
+  // Word q's count of flagged tokens in lower words (thread q; J W <= NT).
+  const uint32_t word = static_cast<int>(threadIdx.x) < J * W ? bits[threadIdx.x] : 0u;
+  uint32_t tot;
+  const uint32_t before = block_excl_scan<NT>(__popc(word), &tot, sh);
+  if (static_cast<int>(threadIdx.x) < J * W) bits[threadIdx.x] = before;
+  __syncthreads();
+  const uint32_t lt = (1u << lane) - 1u;
+  uint32_t out = 0u;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      l = fminf(l, __shfl_xor_sync(0xffffffffu, l, off));
-      h = fmaxf(h, __shfl_xor_sync(0xffffffffu, h, off));
-    }
-    if (lane == 31) sh.bcast[7] = wi;
-    if (lane == 0) {
-      sh.fcast[0] = l;
-      sh.fcast[1] = h;
-    }
+  for (int j = 0; j < E; ++j) {
+    const uint32_t b = __ballot_sync(0xffffffffu, (f >> j) & 1u);
+    if (j < J && ((f >> j) & 1u) && bits[j * W + warp] + __popc(b & lt) < take) out |= 1u << j;
   }
-  __syncthreads();
-  const uint32_t out = sh.warp_b[warp] + incl - v;
-  *total = sh.bcast[7];
-  *lo = sh.fcast[0];
-  *hi = sh.fcast[1];
-  __syncthreads();
+  __syncthreads();  // bits may be reused
   return out;
 }
 
-// One stage over the register-resident tokens: picks the k best (key desc,
-// index asc; NaN keys lowest) among the tokens whose bit is set in elig (bit
-// e: token i0 + e). n_cand candidates in the block, n_nan of them NaN, and
-// nan_before NaN candidates in lower-numbered threads. hist holds the
-// candidates' numbers in bins (kHistCopies copies, built by the caller); scratch is 2048 words
-// that may be overwritten, winmap a zeroed bitmap of ceil(n_past/32) words.
-// Returns the picks as a bit mask. Block-uniform arguments except key, elig,
-// nan_before.
+// One stage over the register-resident tokens: picks the k best (score desc,
+// index asc; NaN lowest) among the tokens whose bit is set in elig (bit j:
+// token j NT + t, score v[j], already free of -0; v is overwritten when the
+// boundary bin is crowded). n_cand candidates in the block, J rows. hist
+// holds the candidates' numbers in bins (kHistCopies copies, built and
+// published by the caller; its total is the number of non-NaN candidates);
+// scratch is 2048 words that may be overwritten, winmap a zeroed bitmap and
+// bits a scratch one (J NT / 32 words each); *list_n (this stage's own
+// count) is 0 on entry. Returns the picks as a bit mask. Block-uniform
+// arguments except v, elig.
 template <int NT, int E>
-__device__ uint32_t stage_reg(const uint32_t (&key)[E], uint32_t elig, int i0, uint32_t k, uint32_t n_cand,
-                              uint32_t n_nan, uint32_t nan_before, Bins bins, const uint32_t* hist,
-                              uint32_t* scratch, uint32_t* list_key, uint32_t* list_idx, uint32_t* winmap,
-                              SelShared& sh) {
+__device__ uint32_t stage_reg(float (&v)[E], uint32_t elig, int J, uint32_t k, uint32_t n_cand, Bins bins,
+                              const uint32_t* hist, uint32_t* scratch, uint32_t* list_key, uint32_t* list_idx,
+                              uint32_t* list_n, uint32_t* winmap, uint32_t* bits, SelShared& sh) {
+  constexpr int W = NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (k == 0u) return 0u;
   if (k >= n_cand) return elig;
-  const uint32_t n_num = n_cand - n_nan;
   uint32_t pick = 0u;
+  // The boundary bin holds the scores in [v_lo, v_hi) (NaN fails both tests).
+  uint32_t bsel, above, cnt_b, n_num;
+  float v_lo = 0.0f, v_hi = 0.0f;
+  boundary_bin<NT, kHistCopies>(hist, k, sh, &bsel, &above, &cnt_b, &bins, &v_lo, &v_hi, &n_num);
   if (k > n_num) {  // every number, then the lowest-index NaNs
-    const uint32_t take = k - n_num;
-    uint32_t r = nan_before;
+    uint32_t nan = 0u;
 #pragma unroll
-    for (int e = 0; e < E; ++e) {
-      if (!((elig >> e) & 1u)) continue;
-      if (key[e] != kNanKey) {
-        pick |= 1u << e;
-      } else {
-        if (r < take) pick |= 1u << e;
-        ++r;
-      }
+    for (int j = 0; j < E; ++j) {
+      const uint32_t el = (elig >> j) & 1u;
+      const uint32_t num = v[j] == v[j] ? 1u : 0u;
+      pick |= (el & num) << j;
+      nan |= (el & (num ^ 1u)) << j;
     }
-    return pick;
+    return pick | lowest_index<NT, E>(nan, k - n_num, J, bits, sh);
   }
-  uint32_t bsel, above, cnt_b;
-  boundary_bin<NT, kHistCopies>(hist, k, sh, &bsel, &above, &cnt_b);
   uint32_t k_rem = k - above;
   if (bsel != kNoBin && cnt_b == k_rem) {  // the whole boundary bin is taken
 #pragma unroll
-    for (int e = 0; e < E; ++e)
-      if (((elig >> e) & 1u) && key[e] != kNanKey && bins.of(key_value(key[e])) >= static_cast<int>(bsel))
-        pick |= 1u << e;
+    for (int j = 0; j < E; ++j) pick |= (((elig >> j) & 1u) & (v[j] >= v_lo ? 1u : 0u)) << j;
     return pick;
   }
   if (bsel != kNoBin && cnt_b <= static_cast<uint32_t>(NT)) {
-    if (threadIdx.x == 0) sh.list_n = 0u;
-    __syncthreads();
     uint32_t in_bin = 0u;
 #pragma unroll
-    for (int e = 0; e < E; ++e) {
-      if (!((elig >> e) & 1u) || key[e] == kNanKey) continue;
-      const int b = bins.of(key_value(key[e]));
-      if (b > static_cast<int>(bsel)) {
-        pick |= 1u << e;
-      } else if (b == static_cast<int>(bsel)) {
-        in_bin |= 1u << e;
-        const uint32_t j = atomicAdd(&sh.list_n, 1u);
-        if (j < static_cast<uint32_t>(NT)) {
-          list_key[j] = key[e];
-          list_idx[j] = static_cast<uint32_t>(i0 + e);
+    for (int j = 0; j < E; ++j) {
+      const uint32_t el = (elig >> j) & 1u;
+      const uint32_t up = v[j] >= v_hi ? 1u : 0u;
+      pick |= (el & up) << j;
+      in_bin |= (el & (v[j] >= v_lo ? 1u : 0u) & (up ^ 1u)) << j;
+    }
+    // The boundary bin's candidates go to the list, one atomic per thread.
+    if (in_bin) {
+      uint32_t q = atomicAdd(list_n, static_cast<uint32_t>(__popc(in_bin)));
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        if (!((in_bin >> j) & 1u)) continue;
+        if (q < static_cast<uint32_t>(NT)) {
+          list_key[q] = __float_as_uint(v[j]);
+          list_idx[q] = static_cast<uint32_t>(j * NT) + threadIdx.x;
+        }
+        ++q;
+      }
+    }
+    __syncthreads();
+    const uint32_t m = min(*list_n, static_cast<uint32_t>(NT));
+    // 2^lg threads rank one candidate (2^lg m <= NT, 2^lg <= 32, aligned
+    // within a warp), each against every 2^lg-th other one, then sum over
+    // those lanes. The candidates are numbers, so float order is key order.
+    int lg = 5;
+    while (lg > 0 && (m << lg) > static_cast<uint32_t>(NT)) --lg;
+    const uint32_t cand = threadIdx.x >> lg, sub = threadIdx.x & ((1u << lg) - 1u);
+    if ((threadIdx.x & ~31u) < (m << lg)) {  // warps holding a candidate
+      uint32_t rank = 0u, it = 0u;
+      if (cand < m) {
+        const float kt = __uint_as_float(list_key[cand]);
+        it = list_idx[cand];
+        for (uint32_t q = sub; q < m; q += 1u << lg) {
+          const float kq = __uint_as_float(list_key[q]);
+          rank += (kq > kt || (kq == kt && list_idx[q] < it)) ? 1u : 0u;
         }
       }
+      for (int off = (1 << lg) >> 1; off > 0; off >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off);
+      if (cand < m && sub == 0u && rank < k_rem) atomicOr(&winmap[it >> 5], 1u << (it & 31));
     }
     __syncthreads();
-    const uint32_t m = min(sh.list_n, static_cast<uint32_t>(NT));
-    // T threads rank one candidate (T m <= NT, T <= 32, aligned within a
-    // warp), each against every T-th other one, then sum over the T lanes.
-    uint32_t T = 32u;
-    while (T > 1u && T * m > static_cast<uint32_t>(NT)) T >>= 1;
-    const uint32_t cand = threadIdx.x / T, sub = threadIdx.x % T;
-    uint32_t rank = 0u, kt = 0u, it = 0u;
-    if (cand < m) {
-      kt = list_key[cand];
-      it = list_idx[cand];
-      for (uint32_t j = sub; j < m; j += T) {
-        const uint32_t kj = list_key[j];
-        rank += (kj > kt || (kj == kt && list_idx[j] < it)) ? 1u : 0u;
-      }
-    }
-    for (uint32_t off = T >> 1; off > 0u; off >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off);
-    if (cand < m && sub == 0u && rank < k_rem) atomicOr(&winmap[it >> 5], 1u << (it & 31));
-    __syncthreads();
+    if (in_bin) {
 #pragma unroll
-    for (int e = 0; e < E; ++e) {
-      if (!((in_bin >> e) & 1u)) continue;
-      const int i = i0 + e;
-      if ((winmap[i >> 5] >> (i & 31)) & 1u) pick |= 1u << e;
+      for (int j = 0; j < E; ++j)
+        if (((in_bin >> j) & 1u) && ((winmap[j * W + warp] >> lane) & 1u)) pick |= 1u << j;
     }
     return pick;
   }
-  // Boundary bin too crowded: exact search over integer key windows.
+  // Boundary bin too crowded (or no bin: cannot happen): exact search over
+  // integer score keys. The scores turn into their keys in place (the
+  // caller's array is not read after the stage), so that no second array
+  // holds registers.
+#pragma unroll
+  for (int j = 0; j < E; ++j) v[j] = __uint_as_float(score_key(v[j]));
   uint32_t lo = 2u, hi = kTaken - 1u, cnt = n_num;
   if (bsel != kNoBin) {
+    const uint32_t key_lo = score_key(v_lo), key_hi = v_hi == v_hi ? score_key(v_hi) : kTaken;
     uint32_t blo = 0xFFFFFFFFu, bhi = 0u;
 #pragma unroll
-    for (int e = 0; e < E; ++e) {
-      if (!((elig >> e) & 1u) || key[e] == kNanKey) continue;
-      if (bins.of(key_value(key[e])) == static_cast<int>(bsel)) {
-        blo = min(blo, key[e]);
-        bhi = max(bhi, key[e]);
+    for (int j = 0; j < E; ++j) {
+      const uint32_t x = __float_as_uint(v[j]);
+      if (((elig >> j) & 1u) && x >= key_lo && x < key_hi) {
+        blo = min(blo, x);
+        bhi = max(bhi, x);
       }
     }
     block_minmax<NT>(blo, bhi, &lo, &hi, sh);
@@ -1033,22 +1142,22 @@ __device__ uint32_t stage_reg(const uint32_t (&key)[E], uint32_t elig, int i0, u
   }
   for (int round = 0; round < 8; ++round) {
     if (lo == hi) break;
-    const uint64_t W = static_cast<uint64_t>(hi - lo) + 1u;
+    const uint64_t Wd = static_cast<uint64_t>(hi - lo) + 1u;
     for (int b = threadIdx.x; b < kSelectBins; b += NT) scratch[b] = 0u;
     __syncthreads();
 #pragma unroll
-    for (int e = 0; e < E; ++e) {
-      const uint32_t x = key[e];
-      if (((elig >> e) & 1u) && x >= lo && x <= hi)
-        atomicAdd(&scratch[(static_cast<uint64_t>(x - lo) * kSelectBins) / W], 1u);
+    for (int j = 0; j < E; ++j) {
+      const uint32_t x = __float_as_uint(v[j]);
+      if (((elig >> j) & 1u) && x >= lo && x <= hi)
+        atomicAdd(&scratch[(static_cast<uint64_t>(x - lo) * kSelectBins) / Wd], 1u);
     }
     __syncthreads();
     uint32_t b2, above2, cnt2;
     boundary_bin<NT>(scratch, k_rem, sh, &b2, &above2, &cnt2);
     if (b2 == kNoBin) break;  // fewer candidates than k_rem: cannot happen
     k_rem -= above2;
-    const uint32_t lo_b = lo + static_cast<uint32_t>((b2 * W + kSelectBins - 1) / kSelectBins);
-    const uint32_t hi_b = lo + static_cast<uint32_t>(((b2 + 1) * W + kSelectBins - 1) / kSelectBins) - 1u;
+    const uint32_t lo_b = lo + static_cast<uint32_t>((b2 * Wd + kSelectBins - 1) / kSelectBins);
+    const uint32_t hi_b = lo + static_cast<uint32_t>(((b2 + 1) * Wd + kSelectBins - 1) / kSelectBins) - 1u;
     if (cnt2 == k_rem) {  // the whole window bin is taken: winners are keys >= lo_b
       lo = hi = lo_b - 1u;
       cnt = 0u;
@@ -1063,118 +1172,153 @@ __device__ uint32_t stage_reg(const uint32_t (&key)[E], uint32_t elig, int i0, u
   // (cnt of them; all when k_rem == cnt).
   uint32_t eq = 0u;
 #pragma unroll
-  for (int e = 0; e < E; ++e) {
-    if (!((elig >> e) & 1u)) continue;
-    if (key[e] > lo) pick |= 1u << e;
-    if (key[e] == lo) eq |= 1u << e;
+  for (int j = 0; j < E; ++j) {
+    const uint32_t el = (elig >> j) & 1u;
+    const uint32_t x = __float_as_uint(v[j]);
+    pick |= (el & (x > lo ? 1u : 0u)) << j;
+    eq |= (el & (x == lo ? 1u : 0u)) << j;
   }
-  uint32_t tot;
-  uint32_t r = block_excl_scan<NT>(__popc(eq), &tot, sh);
-#pragma unroll
-  for (int e = 0; e < E; ++e) {
-    if (!((eq >> e) & 1u)) continue;
-    if (r < k_rem) pick |= 1u << e;
-    ++r;
-  }
-  return pick;
+  return pick | lowest_index<NT, E>(eq, k_rem, J, bits, sh);
 }
 
+// Clears what select_slab_reg accumulates into (both histograms, both winner
+// bitmaps, the list counts); needs no input, so the selection kernel runs it
+// before it waits for the scores.
 template <int NT, int E>
+__device__ void select_reg_clear(uint32_t* smem, SelShared& sh) {
+  constexpr int kWords = E * NT / 32;
+  uint4* h4 = reinterpret_cast<uint4*>(smem);  // 16-byte aligned
+  for (int b = threadIdx.x; b < 2 * kHistCopies * kSelectBins / 4; b += NT) h4[b] = make_uint4(0u, 0u, 0u, 0u);
+  uint32_t* win = smem + 2 * kHistCopies * kSelectBins + 2 * NT;
+  for (int b = threadIdx.x; b < 2 * kWords; b += NT) win[b] = 0u;
+  if (threadIdx.x < 2) sh.list_cnt[threadIdx.x] = 0u;
+  __syncthreads();
+}
+
+// CLEARED: the caller ran select_reg_clear on smem since its last use.
+template <int NT, int E, bool CLEARED = false>
 __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, SelShared& sh) {
+  static_assert(E <= 32, "rows are bits of a word");
+  constexpr int W = NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int n_past = static_cast<int>(a.n_tokens - a.rp);
-  const int words = (n_past + 31) / 32;
+  const int J = (n_past + NT - 1) / NT;  // rows, <= E
   uint32_t* hist_t = smem;
   uint32_t* hist_v = hist_t + kHistCopies * kSelectBins;
   uint32_t* list_key = hist_v + kHistCopies * kSelectBins;
   uint32_t* list_idx = list_key + NT;
   uint32_t* win_t = list_idx + NT;
-  uint32_t* win_v = win_t + words;
-  const int copy = ((threadIdx.x >> 5) % kHistCopies) * kSelectBins;  // this warp's histogram copy
+  uint32_t* win_v = win_t + E * W;
+  uint32_t* bits = win_v + E * W;
+  const int copy = (warp % kHistCopies) * kSelectBins;  // this warp's histogram copy
   const float* tar = a.tar + s * a.n_tokens;
   const float* van = a.van + s * a.n_tokens;
-  const int chunk = (n_past + NT - 1) / NT;  // <= E
-  const int i0 = min(n_past, static_cast<int>(threadIdx.x) * chunk);
-  const int cnt = min(n_past - i0, chunk);
-  const uint32_t mine = cnt >= 32 ? 0xFFFFFFFFu : ((1u << cnt) - 1u);
+  // fma(x, sign, 0) applies the ablation's sign and turns -0 into +0 (NaN stays NaN).
+  const float sgn_t = a.neg_tar ? -1.0f : 1.0f, sgn_v = a.neg_van ? -1.0f : 1.0f;
+  if (!CLEARED) select_reg_clear<NT, E>(smem, sh);
 
-  for (int b = threadIdx.x; b < 2 * kHistCopies * kSelectBins; b += NT) hist_t[b] = 0u;  // histograms
-  for (int b = threadIdx.x; b < 2 * words; b += NT) win_t[b] = 0u;                          // bitmaps
-  __syncthreads();
-
-  // Keys, TaR histogram, range of VaN. A warp's chunks are contiguous, so the
-  // loads of one e across the warp share cache lines (plain loads through L1).
-  // All of a thread's loads are issued before any result is used.
-  uint32_t tk[E], vk[E];
-#pragma unroll
-  for (int e = 0; e < E; ++e) {
-    tk[e] = e < cnt ? __float_as_uint(tar[i0 + e]) : 0u;
-    vk[e] = e < cnt ? __float_as_uint(van[i0 + e]) : 0u;
-  }
-  uint32_t nan_t = 0u;
-  float vmin = INFINITY, vmax = -INFINITY;
+  // Scores (a batch's loads issued before any is used), TaR histogram, VaN
+  // range.
+  float tv[E], vv[E];
+  const int rows_mine = n_past > static_cast<int>(threadIdx.x) ? (n_past - 1 - static_cast<int>(threadIdx.x)) / NT + 1 : 0;
+  const uint32_t mine = rows_mine >= 32 ? 0xFFFFFFFFu : ((1u << rows_mine) - 1u);
+  float vmin = INFINITY, vmax = -INFINITY;  // fminf / fmaxf pass over NaN
   const Bins bt = tar_bins();
+  constexpr int kB = E < 8 ? E : 8;
 #pragma unroll
-  for (int e = 0; e < E; ++e) {
-    const float t = __uint_as_float(tk[e]), u = __uint_as_float(vk[e]);
-    const float tv = (a.neg_tar ? -t : t) + 0.0f;  // NaN stays NaN, -0 becomes +0
-    const float vv = (a.neg_van ? -u : u) + 0.0f;
-    tk[e] = e < cnt ? score_key(tv) : kNanKey;
-    vk[e] = e < cnt ? score_key(vv) : kNanKey;
-    if (e < cnt) {
-      if (tv == tv) {
-        atomicAdd(&hist_t[copy + bt.of(tv)], 1u);
-      } else {
-        ++nan_t;
-      }
-      if (vv == vv) {
-        vmin = fminf(vmin, vv);
-        vmax = fmaxf(vmax, vv);
+  for (int j0 = 0; j0 < E; j0 += kB) {
+#pragma unroll
+    for (int j = j0; j < j0 + kB && j < E; ++j) {
+      const bool ok = (mine >> j) & 1u;
+      tv[j] = ok ? __ldcg(tar + j * NT + threadIdx.x) : 0.0f;
+      vv[j] = ok ? __ldcg(van + j * NT + threadIdx.x) : 0.0f;
+    }
+#pragma unroll
+    for (int j = j0; j < j0 + kB && j < E; ++j) {
+      tv[j] = fmaf(tv[j], sgn_t, 0.0f);
+      vv[j] = fmaf(vv[j], sgn_v, 0.0f);
+      if ((mine >> j) & 1u) {
+        if (tv[j] == tv[j]) atomicAdd(&hist_t[copy + bt.of(tv[j])], 1u);
+        vmin = fminf(vmin, vv[j]);
+        vmax = fmaxf(vmax, vv[j]);
       }
     }
   }
-  uint32_t nan_t_all;
-  const uint32_t nan_t_before = block_scan_minmax<NT>(nan_t, &nan_t_all, &vmin, &vmax, sh);
+  // The warps' parts of the VaN range go out with the barrier that
+  // publishes the TaR histogram (nothing else writes warp_f / warp_g here).
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, off));
+    vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, off));
+  }
+  if (lane == 0) {
+    sh.warp_f[warp] = vmin;
+    sh.warp_g[warp] = vmax;
+  }
+  __syncthreads();
+  vmin = lane < W ? sh.warp_f[lane] : INFINITY;
+  vmax = lane < W ? sh.warp_g[lane] : -INFINITY;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, off));
+    vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, off));
+  }
   const Bins bv = range_bins(vmin, vmax);
+  float* vstash = reinterpret_cast<float*>(bits + E * W);
+  if (E > kRegStashRows) {
+#pragma unroll
+    for (int j = 0; j < E; ++j)
+      if ((mine >> j) & 1u) vstash[j * NT + threadIdx.x] = vv[j];
+  }
 
   // TaR stage over all past tokens.
-  const uint32_t pick_t = stage_reg<NT, E>(tk, mine, i0, static_cast<uint32_t>(a.n_tar),
-                                           static_cast<uint32_t>(n_past), nan_t_all, nan_t_before, bt, hist_t,
-                                           hist_t, list_key, list_idx, win_t, sh);
+  const uint32_t pick_t = stage_reg<NT, E>(tv, mine, J, static_cast<uint32_t>(a.n_tar),
+                                           static_cast<uint32_t>(n_past), bt, hist_t, hist_t, list_key, list_idx,
+                                           &sh.list_cnt[0], win_t, bits, sh);
+  if (E > kRegStashRows) {  // each thread reads back only what it stored
+#pragma unroll
+    for (int j = 0; j < E; ++j) vv[j] = ((mine >> j) & 1u) ? vstash[j * NT + threadIdx.x] : 0.0f;
+  }
   // VaN histogram of the tokens TaR left.
   const uint32_t rest = mine & ~pick_t;
-  uint32_t nan_v = 0u;
 #pragma unroll
-  for (int e = 0; e < E; ++e) {
-    if (!((rest >> e) & 1u)) continue;
-    if (vk[e] != kNanKey) {
-      atomicAdd(&hist_v[copy + bv.of(key_value(vk[e]))], 1u);
-    } else {
-      ++nan_v;
-    }
-  }
-  uint32_t nan_v_all;
-  float d0 = 0.0f, d1 = 0.0f;
-  const uint32_t nan_v_before = block_scan_minmax<NT>(nan_v, &nan_v_all, &d0, &d1, sh);
+  for (int j = 0; j < E; ++j)
+    if (((rest >> j) & 1u) && vv[j] == vv[j]) atomicAdd(&hist_v[copy + bv.of(vv[j])], 1u);
+  __syncthreads();  // publishes the histogram; the TaR stage's list has been read
 
   // VaN stage over the past tokens TaR left.
-  const uint32_t pick_v = stage_reg<NT, E>(vk, rest, i0, static_cast<uint32_t>(a.n_van),
-                                           static_cast<uint32_t>(n_past - a.n_tar), nan_v_all, nan_v_before, bv,
-                                           hist_v, hist_t, list_key, list_idx, win_v, sh);
+  const uint32_t pick_v = stage_reg<NT, E>(vv, rest, J, static_cast<uint32_t>(a.n_van),
+                                           static_cast<uint32_t>(n_past - a.n_tar), bv, hist_v, hist_t, list_key,
+                                           list_idx, &sh.list_cnt[1], win_v, bits, sh);
 
-  // Ascending kept indices: this thread's picks at the block prefix of the
-  // counts, then the recent frames.
+  // Ascending kept indices: a pick's position is the number of picks of
+  // lower index (warp w's ballot over row j is word j W + w of the picks'
+  // bitmap, and word order is index order), so each row's picks of a warp
+  // are stored to consecutive positions; the recent frames follow.
   const uint32_t pick = pick_t | pick_v;
-  uint32_t total;
-  uint32_t pos = block_excl_scan<NT>(__popc(pick), &total, sh);
-  int32_t* kept = a.kept + s * a.budget;
 #pragma unroll
-  for (int e = 0; e < E; ++e) {
-    if (!((pick >> e) & 1u)) continue;
-    if (pos < a.budget) kept[pos] = i0 + e;
-    ++pos;
+  for (int j = 0; j < E; ++j) {
+    const uint32_t b = __ballot_sync(0xffffffffu, (pick >> j) & 1u);
+    if (j < J && lane == 0) bits[j * W + warp] = b;
   }
-  // total == n_tar + n_van by construction; the guards only keep a broken
-  // count from writing outside this slab's row.
+  __syncthreads();
+  const uint32_t word = static_cast<int>(threadIdx.x) < J * W ? bits[threadIdx.x] : 0u;
+  uint32_t total;
+  const uint32_t before = block_excl_scan<NT>(__popc(word), &total, sh);
+  if (static_cast<int>(threadIdx.x) < J * W) win_t[threadIdx.x] = before;  // the TaR winners are read
+  __syncthreads();
+  // total == n_tar + n_van and total + rp == budget by construction; the
+  // bounds only keep a broken count from writing outside this slab's row.
+  int32_t* kept = a.kept + s * a.budget;
+  const uint32_t lt = (1u << lane) - 1u;
+#pragma unroll
+  for (int j = 0; j < E; ++j) {
+    const uint32_t b = __ballot_sync(0xffffffffu, (pick >> j) & 1u);
+    if ((pick >> j) & 1u) {
+      const uint32_t at = win_t[j * W + warp] + __popc(b & lt);
+      if (at < a.budget) kept[at] = static_cast<int32_t>(j * NT + threadIdx.x);
+    }
+  }
   for (int64_t j = threadIdx.x; j < a.rp; j += NT)
     if (total + j < a.budget) kept[total + j] = static_cast<int32_t>(n_past + j);
   __syncthreads();  // the block's shared memory may be reused for the next slab

@@ -8,27 +8,34 @@ namespace ipv {
 namespace {
 
 __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a) {
-  extern __shared__ uint32_t sm_sel[];
+  extern __shared__ __align__(16) uint32_t sm_sel[];
   __shared__ dev::SelShared sh;
   pdl_trigger();
   pdl_wait();  // the scores come from the scoring kernel
   dev::select_slab<kSelectThreads>(a, blockIdx.x, sm_sel, sh);
 }
 
-// The same selection with every thread's share of the keys in registers
-// (at most E past tokens per thread).
+// The same selection with every thread's share of the scores in registers
+// (at most E past tokens per thread). Its shared memory is cleared before it
+// waits for the scoring kernel.
 template <int E>
 __global__ void __launch_bounds__(kSelectThreads, 1) select_reg_kernel(SelectArgs a) {
-  extern __shared__ uint32_t sm_sel[];
+  extern __shared__ __align__(16) uint32_t sm_sel[];
   __shared__ dev::SelShared sh;
   pdl_trigger();
+  dev::select_reg_clear<kSelectThreads, E>(sm_sel, sh);
   pdl_wait();  // the scores come from the scoring kernel
-  dev::select_slab_reg<kSelectThreads, E>(a, blockIdx.x, sm_sel, sh);
+  dev::select_slab_reg<kSelectThreads, E, true>(a, blockIdx.x, sm_sel, sh);
 }
 #ifndef IPV_SELECT_REG_SMALL_E
 #define IPV_SELECT_REG_SMALL_E 10
 #endif
 constexpr int kSelectRegSmallE = IPV_SELECT_REG_SMALL_E;  // fewer registers when a slab needs no more
+
+template <int E>
+constexpr size_t reg_smem_bytes() {
+  return dev::select_reg_smem_words<kSelectThreads, E>() * sizeof(uint32_t);
+}
 
 __global__ void passthrough_kernel(int32_t* kept, int64_t n_slabs, int64_t n_tokens,
                                    int64_t budget) {
@@ -84,23 +91,22 @@ cudaError_t select_prepare(int64_t max_tokens) {
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(select_smem_bytes(max_tokens)));
   if (e != cudaSuccess) return e;
-  const int reg_smem =
-      static_cast<int>(dev::select_reg_smem_words<kSelectThreads>(kSelectThreads * kSelectRegE) * sizeof(uint32_t));
   e = cudaFuncSetAttribute(select_reg_kernel<kSelectRegSmallE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           reg_smem);
+                           static_cast<int>(reg_smem_bytes<kSelectRegSmallE>()));
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(select_reg_kernel<kSelectRegE>, cudaFuncAttributeMaxDynamicSharedMemorySize, reg_smem);
+  return cudaFuncSetAttribute(select_reg_kernel<kSelectRegE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(reg_smem_bytes<kSelectRegE>()));
 }
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st) {
   SelectArgs b = a;
   const int64_t n_past = a.n_tokens - a.rp;
   if (n_past <= static_cast<int64_t>(kSelectThreads) * kSelectRegE) {
-    const size_t smem = dev::select_reg_smem_words<kSelectThreads>(n_past) * sizeof(uint32_t);
     if (n_past <= static_cast<int64_t>(kSelectThreads) * kSelectRegSmallE)
-      return launch(select_reg_kernel<kSelectRegSmallE>, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st,
-                    true, b);
-    return launch(select_reg_kernel<kSelectRegE>, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st, true, b);
+      return launch(select_reg_kernel<kSelectRegSmallE>, static_cast<unsigned>(a.n_slabs), kSelectThreads,
+                    reg_smem_bytes<kSelectRegSmallE>(), st, true, b);
+    return launch(select_reg_kernel<kSelectRegE>, static_cast<unsigned>(a.n_slabs), kSelectThreads,
+                  reg_smem_bytes<kSelectRegE>(), st, true, b);
   }
   b.van_smem = van_fits(n_past) ? 1 : 0;
   const size_t smem = dev::select_smem_words<kSelectThreads>(n_past, b.van_smem != 0) * sizeof(uint32_t);

@@ -389,7 +389,7 @@ size_t window_smem_bytes(int qmax, int D, int elem, int r, int64_t n_past) {
   const size_t rec = static_cast<size_t>(r) * qmax;  // recent rows of one score item
   const size_t stream_b = 2 * rec * D * elem + static_cast<size_t>(qmax) * (D + 4) * sizeof(float) +
                           rec * sizeof(float);
-  const size_t owner_b = dev::select_reg_smem_words<kWinThreads>(n_past) * sizeof(uint32_t);
+  const size_t owner_b = dev::select_reg_smem_words<kWinThreads, kWinRegE>() * sizeof(uint32_t);
   return stream_b > owner_b ? stream_b : owner_b;
 }
 
