@@ -569,7 +569,8 @@ __device__ void block_minmax(uint32_t lo, uint32_t hi, uint32_t* out_lo, uint32_
 }
 
 // The bin holding the k-th largest candidate (bins scanned from the top;
-// thread t owns the 2048/NT bins just below bin 2048 - t 2048/NT), the count
+// thread t owns the 2048/NT bins just below bin 2048 - t 2048/NT; hist
+// 16-byte aligned), the count
 // of candidates in higher bins and the bin's own count. kNoBin if the
 // histogram holds fewer than k.
 // COPIES > 1: the histogram is that many copies of 2048 bins, summed here.
@@ -588,12 +589,29 @@ __device__ void boundary_bin(const uint32_t* hist, uint32_t k, SelShared& sh, ui
   const int top = kSelectBins - 1 - BPT * static_cast<int>(threadIdx.x);
   uint32_t h[BPT], local = 0u;
 #pragma unroll
-  for (int j = 0; j < BPT; ++j) {
-    h[j] = 0u;
+  for (int j = 0; j < BPT; ++j) h[j] = 0u;
+  // A thread's bins are adjacent: one vector load per copy (no bank conflict
+  // between lanes, which are BPT words apart).
 #pragma unroll
-    for (int c = 0; c < COPIES; ++c) h[j] += hist[c * kSelectBins + top - j];
-    local += h[j];
+  for (int c = 0; c < COPIES; ++c) {
+    const uint32_t* hc = hist + c * kSelectBins + top - (BPT - 1);
+    if constexpr (BPT == 2) {
+      const uint2 x = *reinterpret_cast<const uint2*>(hc);
+      h[0] += x.y;
+      h[1] += x.x;
+    } else if constexpr (BPT == 4) {
+      const uint4 x = *reinterpret_cast<const uint4*>(hc);
+      h[0] += x.w;
+      h[1] += x.z;
+      h[2] += x.y;
+      h[3] += x.x;
+    } else {
+#pragma unroll
+      for (int j = 0; j < BPT; ++j) h[j] += hc[BPT - 1 - j];
+    }
   }
+#pragma unroll
+  for (int j = 0; j < BPT; ++j) local += h[j];
   const uint32_t incl = warp_incl_scan(local);
   if (lane == 31) sh.warp_a[warp] = incl;
   __syncthreads();

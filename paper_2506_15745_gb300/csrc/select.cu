@@ -37,13 +37,18 @@ constexpr size_t reg_smem_bytes() {
   return dev::select_reg_smem_words<kSelectThreads, E>() * sizeof(uint32_t);
 }
 
+// The index rows of the index kernels below are the same for every slab:
+// block (x, y) computes columns j = x 256 + t, ... once and stores them to
+// rows y, y + gridDim.y, ... (coalesced along j, no division per element).
+constexpr int kIndexThreads = 256;
+constexpr int64_t kIndexRowBlocks = 32;
+
 __global__ void passthrough_kernel(int32_t* kept, int64_t n_slabs, int64_t n_tokens,
                                    int64_t budget) {
-  const int64_t total = n_slabs * budget;
-  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total;
-       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t j = g % budget;
-    kept[g] = j < n_tokens ? static_cast<int32_t>(j) : -1;
+  for (int64_t j = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; j < budget;
+       j += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int32_t v = j < n_tokens ? static_cast<int32_t>(j) : -1;
+    for (int64_t row = blockIdx.y; row < n_slabs; row += gridDim.y) kept[row * budget + j] = v;
   }
 }
 
@@ -54,24 +59,26 @@ __global__ void passthrough_kernel(int32_t* kept, int64_t n_slabs, int64_t n_tok
 __global__ void uniform_kernel(int32_t* kept, int64_t units, int64_t n_frames, int p, int64_t k) {
   pdl_trigger();
   const int64_t per = k * p;
-  const int64_t total = units * per;
-  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total;
-       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t j = g % per;
+  for (int64_t j = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; j < per;
+       j += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int64_t a = j / p;
     const int64_t f = n_frames - 1 - ((k - 1 - a) * n_frames) / k;
-    kept[g] = static_cast<int32_t>(f * p + (j - a * p));
+    const int32_t v = static_cast<int32_t>(f * p + (j - a * p));
+    for (int64_t row = blockIdx.y; row < units; row += gridDim.y) kept[row * per + j] = v;
   }
+}
+
+dim3 index_grid(int64_t rows, int64_t cols) {
+  const int64_t bx = (cols + kIndexThreads - 1) / kIndexThreads;
+  return dim3(static_cast<unsigned>(bx < 4096 ? bx : 4096),
+              static_cast<unsigned>(rows < kIndexRowBlocks ? rows : kIndexRowBlocks));
 }
 
 }  // namespace
 
 cudaError_t launch_uniform(int32_t* kept, int64_t units, int64_t n_tokens, int p, int64_t budget,
                            cudaStream_t st) {
-  const int64_t total = units * budget;
-  const int64_t blocks = (total + 255) / 256;
-  uniform_kernel<<<static_cast<unsigned>(blocks < 4096 ? blocks : 4096), 256, 0, st>>>(
-      kept, units, n_tokens / p, p, budget / p);
+  uniform_kernel<<<index_grid(units, budget), kIndexThreads, 0, st>>>(kept, units, n_tokens / p, p, budget / p);
   return cudaGetLastError();
 }
 
@@ -115,10 +122,7 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t st) {
 
 cudaError_t launch_passthrough(int32_t* kept, int64_t n_slabs, int64_t n_tokens, int64_t budget,
                                cudaStream_t st) {
-  const int64_t total = n_slabs * budget;
-  const int64_t blocks = (total + 255) / 256;
-  passthrough_kernel<<<static_cast<unsigned>(blocks < 4096 ? blocks : 4096), 256, 0, st>>>(
-      kept, n_slabs, n_tokens, budget);
+  passthrough_kernel<<<index_grid(n_slabs, budget), kIndexThreads, 0, st>>>(kept, n_slabs, n_tokens, budget);
   return cudaGetLastError();
 }
 

@@ -350,6 +350,21 @@ def test_full_config(name):
                w.tar_ratio, pid_valid=False)
 
 
+def test_passthrough_full_shape():
+    """A budget of every cached token at the LLaVA shape (112 slabs x 9408
+    tokens): nothing is evicted, so the pass leaves the cache where it is and
+    the kept indices are 0..N-1, through ipv_compress and ipv_select alike."""
+    w, cache = _device_config("llava", patch_ids=True)
+    N, S = w.n_tokens, w.slabs_per_stream
+    k_before = cache.k_live.clone()
+    check_pass(cache, w.n_layers, w.n_kv_heads, N, w.grid_h, w.grid_w, N, w.tar_ratio, pid_valid=False)
+    assert torch.equal(cache.k_live, k_before)
+    kept = torch.full((S, N), -7, dtype=torch.int32, device="cuda")
+    tar = torch.zeros((S, N), dtype=torch.float32, device="cuda")
+    ipv.select(tar, tar, S, N, w.grid_h, w.grid_w, N, w.tar_ratio, kept)
+    assert torch.equal(kept, torch.arange(N, dtype=torch.int32, device="cuda").expand(S, N))
+
+
 def test_streaming_run():
     """1 h at 1 fps at the LLaVA shape (Algorithm 1's loop): 16 frames
     appended per step through ipv_append_frames (patch ids and frame ids
