@@ -253,6 +253,62 @@ def test_select_exact_when_boundary_bins_overflow():
         assert np.array_equal(to_np(kept), want), (budget, alpha)
 
 
+def _extreme_scores(rng, S, N):
+    """fp32 TaR / VaN rows with infinities, NaN, signed zeros, denormals,
+    values far outside TaR's [-1, 1], VaN ranges far wider than 2048 and
+    values on or next to the selection's bin edges."""
+    f32 = np.float32
+    tar = rng.uniform(-1.0, 1.0, size=(S, N)).astype(f32)
+    van = rng.uniform(0.0, 3.0, size=(S, N)).astype(f32)
+    # 0: VaN log-uniform over 60 decades (bins of width 2^89)
+    van[0] = (10.0 ** rng.uniform(-30, 30, N)).astype(f32)
+    # 1: VaN with +inf and -inf among finite values (no finite range)
+    van[1, ::7] = np.inf
+    van[1, 3::11] = -np.inf
+    # 2: TaR far outside [-1, 1], with infinities and NaN
+    tar[2] = rng.uniform(-3.0, 3.0, N).astype(f32)
+    tar[2, ::13] = np.inf
+    tar[2, 5::17] = -np.inf
+    tar[2, 2::19] = np.nan
+    # 3: denormals and signed zeros
+    tar[3] = (rng.integers(-50, 50, N) * f32(1e-44)).astype(f32)
+    van[3] = (rng.integers(0, 50, N) * f32(1e-44)).astype(f32)
+    tar[3, ::5] = -0.0
+    van[3, 1::5] = -0.0
+    # 4: negative VaN over a wide range (as the Reverse ablation feeds it)
+    van[4] = rng.uniform(-1e6, 1e6, N).astype(f32)
+    # 5: values on TaR's bin edges (b - 1024) / 1024 and one ulp either side
+    e = ((rng.integers(0, 2048, N) - 1024) / 1024.0).astype(f32)
+    step = rng.integers(-1, 2, N)
+    tar[5] = np.where(step < 0, np.nextafter(e, f32(-2)), np.where(step > 0, np.nextafter(e, f32(2)), e))
+    van[5] = (rng.integers(0, 3000, N) / 3.0).astype(f32)
+    # 6: every VaN the same huge value, every TaR -inf
+    van[6] = f32(1e30)
+    tar[6] = -np.inf
+    return tar, van
+
+
+@pytest.mark.parametrize("f", [48, 200, 300])
+def test_select_exact_on_extreme_scores(f):
+    """Step (iii) alone on extreme fp32 scores, at slab sizes that take each
+    selection kernel (scores in registers with 10 and 16 rows, keys in
+    shared memory): bit-exact against the oracle's rule."""
+    rng = np.random.default_rng(100 + f)
+    S, p = 7, 64
+    N = f * p
+    r = oracle.recent_frames(f)
+    init_for(S, N, 64, p, "f32")
+    tar, van = _extreme_scores(rng, S, N)
+    for frac, alpha in [(0.5, 0.5), (0.3, 0.9), (0.8, 0.2), (0.65, 1.0), (0.4, 0.0)]:
+        budget = max(r * p + 1, int(frac * N))
+        kept = torch.empty((S, budget), dtype=torch.int32, device="cuda")
+        ipv.select(torch.from_numpy(tar).cuda(), torch.from_numpy(van).cuda(), S, N, 1, p,
+                   budget, alpha, kept)
+        want = oracle.select(tar.astype(np.float64), van.astype(np.float64), N, p, r, budget,
+                             float(np.float32(alpha)))
+        assert np.array_equal(to_np(kept), want), (f, budget, alpha)
+
+
 def test_fused_selection_fallback_matches_steps():
     """V norms that crowd one bin of the VaN map: the fused pass's 512-thread
     selection takes the exact window search (the step kernels' 1024-thread
