@@ -1001,17 +1001,21 @@ __device__ void select_slab(const SelectArgs& a, int64_t s, uint32_t* smem, SelS
 constexpr int kHistCopies = 4;
 
 // Above this many rows the VaN scores wait out the TaR stage in shared
-// memory, so that the stage has the registers it needs.
-constexpr int kRegStashRows = 10;
+// memory, so that the stage has the registers it needs (always, by
+// default: the selection kernel runs at 48 registers).
+#ifndef IPV_REG_STASH_ROWS
+#define IPV_REG_STASH_ROWS 0
+#endif
+constexpr int kRegStashRows = IPV_REG_STASH_ROWS;
 
 // Shared memory of select_slab_reg: hist_t[kHistCopies][2048],
 // hist_v[kHistCopies][2048], list_key[NT], list_idx[NT], three bitmaps of
 // E NT / 32 words (the two stages' boundary-bin winners, and a scratch one
 // for index-order ranks and the picks) and, above kRegStashRows rows, the
 // VaN scores (E NT words).
-template <int NT, int E>
+template <int NT, int E, bool STASH = (E > kRegStashRows)>
 __host__ __device__ constexpr size_t select_reg_smem_words() {
-  return 2 * kHistCopies * kSelectBins + 2 * NT + 3 * (E * NT / 32) + (E > kRegStashRows ? E * NT : 0);
+  return 2 * kHistCopies * kSelectBins + 2 * NT + 3 * (E * NT / 32) + (STASH ? E * NT : 0);
 }
 
 // The `take` lowest-index tokens among those flagged in f (bit j: token
@@ -1214,7 +1218,8 @@ __device__ void select_reg_clear(uint32_t* smem, SelShared& sh) {
 }
 
 // CLEARED: the caller ran select_reg_clear on smem since its last use.
-template <int NT, int E, bool CLEARED = false>
+// STASH: the VaN scores wait out the TaR stage in shared memory.
+template <int NT, int E, bool CLEARED = false, bool STASH = (E > kRegStashRows)>
 __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, SelShared& sh) {
   static_assert(E <= 32, "rows are bits of a word");
   constexpr int W = NT / 32;
@@ -1283,7 +1288,7 @@ __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, 
   }
   const Bins bv = range_bins(vmin, vmax);
   float* vstash = reinterpret_cast<float*>(bits + E * W);
-  if (E > kRegStashRows) {
+  if (STASH) {
 #pragma unroll
     for (int j = 0; j < E; ++j)
       if ((mine >> j) & 1u) vstash[j * NT + threadIdx.x] = vv[j];
@@ -1293,7 +1298,7 @@ __device__ void select_slab_reg(const SelectArgs& a, int64_t s, uint32_t* smem, 
   const uint32_t pick_t = stage_reg<NT, E>(tv, mine, J, static_cast<uint32_t>(a.n_tar),
                                            static_cast<uint32_t>(n_past), bt, hist_t, hist_t, list_key, list_idx,
                                            &sh.list_cnt[0], win_t, bits, sh);
-  if (E > kRegStashRows) {  // each thread reads back only what it stored
+  if (STASH) {  // each thread reads back only what it stored
 #pragma unroll
     for (int j = 0; j < E; ++j) vv[j] = ((mine >> j) & 1u) ? vstash[j * NT + threadIdx.x] : 0.0f;
   }

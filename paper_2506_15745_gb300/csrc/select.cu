@@ -17,9 +17,16 @@ __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a)
 
 // The same selection with every thread's share of the scores in registers
 // (at most E past tokens per thread). Its shared memory is cleared before it
-// waits for the scoring kernel.
+// waits for the scoring kernel. 48 registers per thread leave room for one
+// compaction block beside each selection block (1024 x 48 + 256 x 64 =
+// 65,536), which copies the recent rows while the selection runs: a few
+// spills cost less than the copy bandwidth a full register file would
+// shut out (LLaVA-OV-7B shape: pass 0.2120 against 0.2155 ms at 64).
+#ifndef IPV_SELECT_MAXNREG
+#define IPV_SELECT_MAXNREG 48
+#endif
 template <int E>
-__global__ void __launch_bounds__(kSelectThreads, 1) select_reg_kernel(SelectArgs a) {
+__global__ void __maxnreg__(IPV_SELECT_MAXNREG) select_reg_kernel(SelectArgs a) {
   extern __shared__ __align__(16) uint32_t sm_sel[];
   __shared__ dev::SelShared sh;
   pdl_trigger();
@@ -28,7 +35,7 @@ __global__ void __launch_bounds__(kSelectThreads, 1) select_reg_kernel(SelectArg
   dev::select_slab_reg<kSelectThreads, E, true>(a, blockIdx.x, sm_sel, sh);
 }
 #ifndef IPV_SELECT_REG_SMALL_E
-#define IPV_SELECT_REG_SMALL_E 10
+#define IPV_SELECT_REG_SMALL_E 9
 #endif
 constexpr int kSelectRegSmallE = IPV_SELECT_REG_SMALL_E;  // fewer registers when a slab needs no more
 
