@@ -309,6 +309,32 @@ def test_select_exact_on_extreme_scores(f):
         assert np.array_equal(to_np(kept), want), (f, budget, alpha)
 
 
+@pytest.mark.parametrize("f", [1170, 1171, 10533, 10534, 18725, 18726])
+def test_select_exact_at_kernel_size_limits(f):
+    """One-token frames, so that the past tokens number exactly 1024 / 1025,
+    9216 / 9217 and 16384 / 16385: the last size each selection kernel takes
+    (every row of every thread full) and the first one of the next.
+    Tied, NaN and signed-zero scores; bit-exact against the oracle."""
+    rng = np.random.default_rng(f)
+    S, p, N = 4, 1, f
+    r = oracle.recent_frames(f)
+    init_for(S, N, 64, p, "f32")
+    tar = (rng.integers(-40, 40, size=(S, N)) / 40).astype(np.float32)
+    van = rng.uniform(0.0, 2.0, size=(S, N)).astype(np.float32)
+    van[:, ::3] = np.round(van[:, ::3], 1)
+    tar[1, ::9] = np.nan
+    van[2, 1::7] = np.nan
+    tar[3, ::2] = -0.0
+    for frac, alpha in [(0.5, 0.5), (0.9, 0.3)]:
+        budget = max(r * p + 1, int(frac * N))
+        kept = torch.empty((S, budget), dtype=torch.int32, device="cuda")
+        ipv.select(torch.from_numpy(tar).cuda(), torch.from_numpy(van).cuda(), S, N, 1, 1,
+                   budget, alpha, kept)
+        want = oracle.select(tar.astype(np.float64), van.astype(np.float64), N, p, r, budget,
+                             float(np.float32(alpha)))
+        assert np.array_equal(to_np(kept), want), (f, budget, alpha)
+
+
 def test_fused_selection_fallback_matches_steps():
     """V norms that crowd one bin of the VaN map: the fused pass's 512-thread
     selection takes the exact window search (the step kernels' 1024-thread
