@@ -99,7 +99,9 @@ typedef struct {
                              patch ids) and whose selection keys fit the registers
                              of one block (n_tokens - r*p <= 9216 past tokens);
                              other calls run the step kernels. Both give
-                             bit-identical results. */
+                             bit-identical results; the fused kernel is the
+                             slower one (a slab's selection outlasts its rows'
+                             stay in L2). */
   int van_pool;           /* 0: the VaN stage ranks raw VaN (Sec. 3.2 s_VaN);
                              1: it ranks layer-adaptive pooled VaN (Sec. 3.2,
                              Algorithm 2); needs single_kernel = 0 and
