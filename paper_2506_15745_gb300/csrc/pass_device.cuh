@@ -703,6 +703,12 @@ __device__ void window_search(const uint32_t* key, int n, uint32_t lo, uint32_t 
   *cnt_eq = cnt;
 }
 
+// Largest boundary bin whose candidates are ranked against each other
+// directly (m^2 / block-size comparisons per thread); a larger one, e.g. the
+// whole-frame ties of frame-level scores, takes the window search over key
+// bits, which is linear in the slab.
+constexpr uint32_t kRankMax = 128;
+
 // How a stage's winners are recognised in the marking pass (block-uniform).
 struct Plan {
   int mode;  // 0 none, 1 every candidate, 2 key threshold, 3 bin threshold (+ pre-marked)
@@ -748,7 +754,7 @@ __device__ Plan plan_stage(uint32_t* key, int n, uint32_t k, uint32_t n_cand, ui
     const int lane = threadIdx.x & 31;
     if (threadIdx.x == 0) sh.list_n = 0u;
     __syncthreads();
-    if (cnt_b <= static_cast<uint32_t>(NT)) {
+    if (cnt_b <= kRankMax) {
       // Collect the boundary bin's candidates (a ballot per warp, one atomic).
       for (int i0 = threadIdx.x - lane; i0 < n; i0 += NT) {  // warp-uniform
         const int i = i0 + lane;
@@ -1088,7 +1094,7 @@ __device__ uint32_t stage_reg(float (&v)[E], uint32_t elig, int J, uint32_t k, u
     for (int j = 0; j < E; ++j) pick |= (((elig >> j) & 1u) & (v[j] >= v_lo ? 1u : 0u)) << j;
     return pick;
   }
-  if (bsel != kNoBin && cnt_b <= static_cast<uint32_t>(NT)) {
+  if (bsel != kNoBin && cnt_b <= kRankMax) {
     uint32_t in_bin = 0u;
 #pragma unroll
     for (int j = 0; j < E; ++j) {
