@@ -74,7 +74,8 @@ def check_ablation_pass(cache, w, N, variant, pid_valid):
     assert_gather_exact(k_src, to_np(cache.k_live), kept_np, B)
     assert_gather_exact(v_src, to_np(cache.v_live), kept_np, B)
     if n_diff == 0:
-        o = oracle.compress_ablation(k_src, v_src, N, gh, gw, r, B, w.tar_ratio, variant, pid_src, fid_src)
+        o = oracle.compress_ablation(k_src, v_src, N, gh, gw, r, B, float(np.float32(w.tar_ratio)), variant,
+                                     pid_src, fid_src)
         assert np.array_equal(o[0], kept_np)
     return n_diff
 

@@ -266,7 +266,7 @@ def check_pooled_pass(cache, w, N, tau, pid_valid):
     want_f = np.take_along_axis(fid_src, kept_np, 1) if fid_src is not None else (kept_np // p)
     assert np.array_equal(pd, want_p.astype(np.uint16)) and np.array_equal(fd, want_f.astype(np.uint32))
     if np.array_equal(ks, ko):
-        o_kept = oracle.compress_pooled(k_src, v_src, N, gh, gw, r, B, w.tar_ratio, tau, H,
+        o_kept = oracle.compress_pooled(k_src, v_src, N, gh, gw, r, B, float(np.float32(w.tar_ratio)), tau, H,
                                         None if pid_src is None else pid_src,
                                         None if fid_src is None else fid_src)[0]
         if n_diff == 0:

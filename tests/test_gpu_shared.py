@@ -110,7 +110,8 @@ def check_shared_pass(cache, w, N, pid_valid, tau=None):
     want_f = np.take_along_axis(fid_src, kept_slab, 1) if fid_src is not None else kept_slab // p
     assert np.array_equal(pd, want_p.astype(np.uint16)) and np.array_equal(fd, want_f.astype(np.uint32))
     if n_diff == 0:
-        o = oracle.compress_shared(k_src, v_src, N, gh, gw, r, B, w.tar_ratio, H, pid_src, fid_src,
+        o = oracle.compress_shared(k_src, v_src, N, gh, gw, r, B, float(np.float32(w.tar_ratio)), H,
+                                   pid_src, fid_src,
                                    tau=tau)
         if tau is None or np.array_equal(o[5], ks):
             assert np.array_equal(o[0], kept_np)
