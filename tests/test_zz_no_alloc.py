@@ -153,3 +153,48 @@ def test_static_passes_a_cache_within_budget_through():
     want[:, :N] = torch.arange(N, dtype=torch.int32)
     assert torch.equal(kept.cpu(), want)
     assert torch.equal(cache.k[1], before)
+
+
+def _random_case(case):
+    """A small seeded shape: element type, heads, head_dim, grid, frames,
+    budget and ratio drawn at random; half the cases come compacted before
+    (past rows shuffled with their patch ids)."""
+    rng = np.random.default_rng(900 + case)
+    dtype = ("bf16", "f32")[int(rng.integers(2))]
+    L, H = int(rng.integers(1, 4)), int(rng.integers(1, 5))
+    D = int(rng.choice((16, 32, 64, 128, 256)))
+    gh, gw = int(rng.integers(1, 10)), int(rng.integers(1, 10))
+    f = int(rng.integers(4, 25))
+    r = oracle.recent_frames(f)
+    budget = int(rng.integers(r * gh * gw + 1, f * gh * gw))
+    alpha = float(np.float32(rng.choice([0.0, 1.0, rng.uniform(0, 1)])))
+    w = synth.Workload(f"random{case}", L, H, D, dtype, gh, gw, f, budget, alpha, seed=case)
+    K, V = synth.host_generate(w)
+    N, p, S = w.n_tokens, w.p, w.slabs_per_stream
+    cache = PingPongCache(S, N, D, dtype, patch_ids=True)
+    shuffled = bool(rng.integers(2))
+    if shuffled:
+        n_past = N - r * p
+        perm = rng.permutation(n_past)
+        K[:, :n_past], V[:, :n_past] = K[:, perm], V[:, perm]
+        pid = np.tile((np.arange(N) % p).astype(np.uint16), (S, 1))
+        pid[:, :n_past] = (perm % p).astype(np.uint16)
+        cache.pid[0] = torch.from_numpy(pid.view(np.int16)).cuda()
+    if dtype == "bf16":
+        cache.k[0] = torch.from_numpy(K.view(np.int16)).cuda().view(torch.bfloat16)
+        cache.v[0] = torch.from_numpy(V.view(np.int16)).cuda().view(torch.bfloat16)
+    else:
+        cache.k[0] = torch.from_numpy(K).cuda()
+        cache.v[0] = torch.from_numpy(V).cuda()
+    return w, cache, shuffled
+
+
+def test_static_matches_compress_on_random_shapes():
+    """40 seeded shapes in a row: each call of the static entry point finds
+    the previous, differently shaped call's leftovers in the shared array."""
+    for case in range(40):
+        w, cache, pid_valid = _random_case(case)
+        (kc, kdc, vdc, pc), (ks, kds, vds, ps) = _run_pair(w, cache, pid_valid)
+        assert torch.equal(kc, ks), case
+        assert torch.equal(kdc, kds) and torch.equal(vdc, vds), case
+        assert torch.equal(pc, ps), case
