@@ -494,7 +494,8 @@ def test_streaming_run():
 
 def test_large_config_sampled():
     """8 streams x 80 layers x 8 KV heads, 32768 -> 24576 tokens (~86 GB of
-    K/V plus the second ping-pong half). 8 sampled slabs checked."""
+    K/V plus the second ping-pong half). 64 sampled slabs checked, 8 from
+    each stream."""
     w = synth.CONFIGS["large"]
     S = w.n_slabs
     need = 2 * 2 * S * w.n_tokens * w.head_dim * 2 + 3 * S * w.n_tokens * 4 + (8 << 30)
@@ -507,7 +508,9 @@ def test_large_config_sampled():
     for st in range(w.n_streams):
         synth.device_generate(w, cache.k[0, st * per:(st + 1) * per],
                               cache.v[0, st * per:(st + 1) * per], stream=st)
-    sample = np.random.default_rng(1).choice(S, 8, replace=False)
+    rng = np.random.default_rng(1)
+    sample = np.sort(np.concatenate([st * per + rng.choice(per, 8, replace=False)
+                                     for st in range(w.n_streams)]))
     try:
         check_pass(cache, w.n_streams * w.n_layers, w.n_kv_heads, w.n_tokens, w.grid_h, w.grid_w,
                    w.budget, w.tar_ratio, pid_valid=False, slabs=sample)
