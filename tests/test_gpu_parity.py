@@ -309,11 +309,13 @@ def test_select_exact_on_extreme_scores(f):
         assert np.array_equal(to_np(kept), want), (f, budget, alpha)
 
 
-@pytest.mark.parametrize("f", [1170, 1171, 10533, 10534, 18725, 18726])
+@pytest.mark.parametrize("f", [1170, 1171, 10533, 10534, 18725, 18726, 32768, 32769])
 def test_select_exact_at_kernel_size_limits(f):
     """One-token frames, so that the past tokens number exactly 1024 / 1025,
-    9216 / 9217 and 16384 / 16385: the last size each selection kernel takes
-    (every row of every thread full) and the first one of the next.
+    9216 / 9217 and 16384 / 16385 (the last size each selection kernel takes,
+    every row of every thread full, and the first one of the next), and
+    28672 / 28673 (the keys-in-shared-memory kernel at the large config's
+    size).
     Tied, NaN and signed-zero scores; bit-exact against the oracle."""
     rng = np.random.default_rng(f)
     S, p, N = 4, 1, f

@@ -3,7 +3,7 @@
 ipv_select and the oracle's selection (Sec. 3.3; Algorithm 1 steps 3-5) get
 the same fp32 TaR and VaN rows and must return the same kept indices, bit for
 bit. Shapes span every selection kernel (past tokens up to 9216, up to 16384
-and above); the scores mix uniform and wide-range values, heavy and
+and above, to 40000); the scores mix uniform and wide-range values, heavy and
 frame-like ties, tight clusters, values over many decades, NaN, infinities,
 signed zeros and all-NaN rows.
 """
@@ -58,7 +58,7 @@ def _case(case):
     rng = np.random.default_rng(70000 + case)
     p = int(rng.choice([1, 2, 4, 16, 64, 196]))
     n_past = int(rng.choice([rng.integers(1, 2000), rng.integers(2000, 9300), rng.integers(9200, 16500),
-                             rng.integers(16300, 20000)]))
+                             rng.integers(16300, 28800), rng.integers(28600, 40000)]))
     f = max(3, (n_past // p) * 8 // 7 + 1)
     if f * p > ipv.MAX_TOKENS:
         f = ipv.MAX_TOKENS // p
