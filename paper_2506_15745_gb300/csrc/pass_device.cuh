@@ -1437,21 +1437,46 @@ __device__ __forceinline__ void gather_range(const GatherArgs& a, int64_t g_begi
 
 // Patch and frame ids of the kept rows, one (slab, j) per thread of the
 // grid: consecutive j of a slab are consecutive threads, so the stores are
-// coalesced (ids travel with their rows, Sec. 3.1 K~ = K[:, I, :]).
+// coalesced (ids travel with their rows, Sec. 3.1 K~ = K[:, I, :]). A
+// thread's kB elements are loaded together (kept indices, then the ids they
+// point to), so it waits for two round trips per batch, not two per element.
 __device__ __forceinline__ void gather_ids(const GatherArgs& a) {
   if (!a.pid_dst && !a.fid_dst) return;
+  constexpr int kB = 4;
   const int64_t total = a.n_slabs * a.budget;
   const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < total; g += step) {
-    const int64_t s = g / a.budget;
-    const int64_t j = g - s * a.budget;
-    const int n = a.heads_per_kept > 1 ? a.kept[(s / a.heads_per_kept) * a.budget + j] : a.kept[g];
-    if (n < 0 || n >= a.cap) continue;
-    const int64_t dst = s * a.cap + j;
-    if (a.pid_dst)
-      a.pid_dst[dst] = a.pid_src ? a.pid_src[s * a.cap + n] : static_cast<uint16_t>(n % a.p);
-    if (a.fid_dst)
-      a.fid_dst[dst] = a.fid_src ? a.fid_src[s * a.cap + n] : static_cast<uint32_t>(n / a.p);
+  for (int64_t g0 = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g0 < total; g0 += kB * step) {
+    int n[kB];
+    int64_t base[kB], j[kB];
+#pragma unroll
+    for (int u = 0; u < kB; ++u) {
+      const int64_t g = g0 + u * step;
+      n[u] = -1;
+      base[u] = 0;
+      j[u] = 0;
+      if (g < total) {
+        const int64_t s = g / a.budget;
+        j[u] = g - s * a.budget;
+        base[u] = s * a.cap;
+        n[u] = a.heads_per_kept > 1 ? a.kept[(s / a.heads_per_kept) * a.budget + j[u]] : a.kept[g];
+      }
+    }
+    uint16_t pv[kB];
+    uint32_t fv[kB];
+#pragma unroll
+    for (int u = 0; u < kB; ++u) {
+      const bool ok = n[u] >= 0 && n[u] < a.cap;
+      pv[u] = 0;
+      fv[u] = 0;
+      if (ok && a.pid_dst) pv[u] = a.pid_src ? a.pid_src[base[u] + n[u]] : static_cast<uint16_t>(n[u] % a.p);
+      if (ok && a.fid_dst) fv[u] = a.fid_src ? a.fid_src[base[u] + n[u]] : static_cast<uint32_t>(n[u] / a.p);
+    }
+#pragma unroll
+    for (int u = 0; u < kB; ++u) {
+      if (n[u] < 0 || n[u] >= a.cap) continue;
+      if (a.pid_dst) a.pid_dst[base[u] + j[u]] = pv[u];
+      if (a.fid_dst) a.fid_dst[base[u] + j[u]] = fv[u];
+    }
   }
 }
 
