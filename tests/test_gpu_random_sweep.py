@@ -34,7 +34,7 @@ from test_gpu_shared import check_shared_pass  # noqa: E402
 MODES = ("heads", "heads_single_kernel", "pooled", "shared", "shared_pooled", "tar_reverse",
          "van_reverse", "tar_frame", "uniform")
 ABLATIONS = ("tar_reverse", "van_reverse", "tar_frame", "uniform")
-N_CASES = 405
+N_CASES = 1005
 N_PASSES = 3
 
 
