@@ -523,6 +523,7 @@ ipv_status ipv_select(const float* tar, const float* van, int64_t n_slabs, int64
   a.budget = budget;
   split_budget(budget, tar_ratio, rp, &a.n_tar, &a.n_van);
   a.kept = kept_idx_out;
+  a.num_sms = g.num_sms;
   prof_begin(2, st);
   cudaError_t e = ipv::launch_select(a, st);
   prof_end(2, st);
@@ -593,6 +594,7 @@ ipv_status ipv_compress(ipv_kv* k, ipv_kv* v, int n_layers, int n_kv_heads, int 
   sa.budget = budget;
   split_budget(budget, tar_ratio, sh.rp, &sa.n_tar, &sa.n_van);
   sa.kept = kept_idx_out;
+  sa.num_sms = g.num_sms;
 
   ipv::GatherArgs ga{};
   ga.k_src = k->buf[k->cur];

@@ -182,6 +182,8 @@ struct SelectArgs {
   int32_t* kept;      // [S][budget]
   int neg_tar, neg_van;  // ablation: the stage ranks its negated scores (the lowest first)
   int van_smem;       // set by launch_select: VaN is read into shared memory with TaR, up front
+  int num_sms;        // > 0: the keys-in-shared-memory selection runs one block per SM, each
+                      // looping over slabs (else one block per slab)
 };
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);

@@ -217,6 +217,7 @@ extern "C" ipv_status ipv_compress_static(ipv_kv* k, ipv_kv* v, ipv_dtype dtype,
   sa.n_tar = share > rp ? share - rp : 0;
   sa.n_van = budget - rp - sa.n_tar;
   sa.kept = kept_idx_out;
+  sa.num_sms = dev->num_sms;
   if ((e = ipv::launch_select(sa, cs)) != cudaSuccess) return cuda_reject(e, "selection kernel");
 
   ipv::GatherArgs ga{};

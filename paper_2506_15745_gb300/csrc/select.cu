@@ -1,18 +1,28 @@
-// Step (iii) of the compression pass: the split-budget selection, one
-// 1024-thread block per (layer, KV head) slab. The algorithm (Sec. 3.3;
-// Algorithm 1 steps 3-5) is dev::select_slab_reg in pass_device.cuh (keys in
-// registers), or dev::select_slab (keys in shared memory) for larger slabs.
+// Step (iii) of the compression pass: the split-budget selection, a
+// 1024-thread block per (layer, KV head) slab (for larger slabs, one block per
+// SM taking slabs in turn). The algorithm (Sec. 3.3; Algorithm 1 steps 3-5)
+// is dev::select_slab_reg in pass_device.cuh (keys in registers), or
+// dev::select_slab (keys in shared memory) for larger slabs.
 #include "pass_device.cuh"
 
 namespace ipv {
 namespace {
 
-__global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a) {
+#ifndef IPV_SELECT_MAXNREG
+#define IPV_SELECT_MAXNREG 48
+#endif
+
+// Slabs blockIdx.x, blockIdx.x + gridDim.x, ...: with one block per SM the
+// whole grid starts at once, so the compaction (launched when every block of
+// this grid has started) puts a block beside each of them and copies the
+// recent rows while the selection runs, as it does beside the register
+// kernel. 48 registers leave it room (1024 x 48 + 256 x 64 = 65,536).
+__global__ void __maxnreg__(IPV_SELECT_MAXNREG) select_kernel(SelectArgs a) {
   extern __shared__ __align__(16) uint32_t sm_sel[];
   __shared__ dev::SelShared sh;
   pdl_trigger();
   pdl_wait();  // the scores come from the scoring kernel
-  dev::select_slab<kSelectThreads>(a, blockIdx.x, sm_sel, sh);
+  for (int64_t s = blockIdx.x; s < a.n_slabs; s += gridDim.x) dev::select_slab<kSelectThreads>(a, s, sm_sel, sh);
 }
 
 // The same selection with every thread's share of the scores in registers
@@ -22,9 +32,6 @@ __global__ void __launch_bounds__(kSelectThreads, 1) select_kernel(SelectArgs a)
 // 65,536), which copies the recent rows while the selection runs: a few
 // spills cost less than the copy bandwidth a full register file would
 // shut out (LLaVA-OV-7B shape: pass 0.2120 against 0.2155 ms at 64).
-#ifndef IPV_SELECT_MAXNREG
-#define IPV_SELECT_MAXNREG 48
-#endif
 template <int E>
 __global__ void __maxnreg__(IPV_SELECT_MAXNREG) select_reg_kernel(SelectArgs a) {
   extern __shared__ __align__(16) uint32_t sm_sel[];
@@ -124,7 +131,8 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t st) {
   }
   b.van_smem = van_fits(n_past) ? 1 : 0;
   const size_t smem = dev::select_smem_words<kSelectThreads>(n_past, b.van_smem != 0) * sizeof(uint32_t);
-  return launch(select_kernel, static_cast<unsigned>(a.n_slabs), kSelectThreads, smem, st, true, b);
+  const int64_t grid = a.num_sms > 0 && a.num_sms < a.n_slabs ? a.num_sms : a.n_slabs;
+  return launch(select_kernel, static_cast<unsigned>(grid), kSelectThreads, smem, st, true, b);
 }
 
 cudaError_t launch_passthrough(int32_t* kept, int64_t n_slabs, int64_t n_tokens, int64_t budget,

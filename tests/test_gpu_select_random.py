@@ -91,3 +91,26 @@ def test_select_matches_oracle_on_random_scores(block):
         else:
             want = oracle.select(tar.astype(np.float64), van.astype(np.float64), N, p, r, budget, alpha)
         assert np.array_equal(got, want), (case, S, N, p, budget, alpha)
+
+
+def test_select_on_more_slabs_than_sms():
+    """Slabs above the register kernels' size, more of them than the GPU has
+    SMs: the keys-in-shared-memory kernel then runs one block per SM, each
+    taking slabs in turn. Every slab must match the oracle."""
+    rng = np.random.default_rng(91)
+    S, p = 300, 4
+    N = 20000
+    r = oracle.recent_frames(N // p)
+    budget = 15001
+    alpha = float(np.float32(0.4))
+    tar, van = _scores(rng, S, N)
+    ipv.init(device=0, dtype="f32", max_head_dim=64, max_frame_tokens=p, max_slabs=S, token_capacity=N)
+    try:
+        kept = torch.empty((S, budget), dtype=torch.int32, device="cuda")
+        ipv.select(torch.from_numpy(tar).cuda(), torch.from_numpy(van).cuda(), S, N, 1, p, budget, alpha, kept)
+        got = kept.cpu().numpy()
+    finally:
+        torch.cuda.synchronize()
+        ipv.shutdown()
+    want = oracle.select(tar.astype(np.float64), van.astype(np.float64), N, p, r, budget, alpha)
+    assert np.array_equal(got, want)
