@@ -74,3 +74,18 @@ def test_workload_strings_fit_the_record():
     """The driver's record keeps 120 characters of config.workload."""
     for w in synth.CONFIGS.values():
         assert len(bench.workload_desc(w)) <= 120, w.name
+
+
+def test_traffic_is_reported_only_for_the_captured_sources(monkeypatch):
+    """The roofline's DRAM traffic comes from the committed ncu capture only
+    while the kernel sources are the ones it was taken on (their digest is
+    stored beside it), and only for its own workload."""
+    with open(os.path.join(ROOT, "profiles", "dram_traffic.json")) as fh:
+        rec = json.load(fh)
+    captured = rec["kernels"]["gather"]["dram_bytes_per_launch_full_size"]
+    monkeypatch.setattr(bench, "source_digest", lambda: rec["source_digest"])
+    assert bench.ncu_traffic("gather", rec["workload"]) == captured
+    assert bench.ncu_traffic("gather", "qwen") is None
+    assert bench.ncu_traffic("no_such_kernel", rec["workload"]) is None
+    monkeypatch.setattr(bench, "source_digest", lambda: "0" * 16)
+    assert bench.ncu_traffic("gather", rec["workload"]) is None
